@@ -1,0 +1,189 @@
+/*
+ * blr.h — C ABI of the GB300 (sm_103a) BD-LRU scan library (libblr.so).
+ *
+ * The BD-LRU of RecBLR (arXiv 2406.12580, Sec. 3.2) is the diagonal, per-channel
+ * linear recurrence
+ *     h_t = alpha_t * h_{t-1} + beta_t * x_t                                (Sec. 3.2, Eq. linrnn)
+ * whose coefficients depend only on the current input through two gates,
+ *     r_t = sigmoid(rho_t),  i_t = sigmoid(iota_t)                          (Sec. 3.2, gate equations)
+ *     alpha_t = exp(-c * softplus(Lambda) * r_t)                            (Sec. 3.2; c = 1 in the paper)
+ *     beta_t  = sqrt(1 - alpha_t^2) * i_t                                   (Sec. 3.2)
+ * where rho_t = W_r x_t + b_r and iota_t = W_i x_t + b_i are the gate logits.
+ * The gate projections are NOT part of this library: callers pass their
+ * pre-activation outputs ("gate_logits"). Lambda is the per-channel learnable
+ * decay parameter; c generalises the paper's exponent (c = 1 reproduces it).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Memory   All pointers except `desc` are DEVICE pointers of the calling
+ *          thread's current CUDA device, owned by the caller. The library never
+ *          allocates, frees or retains memory; inputs are never written.
+ * Layout   Contiguous row-major. x, h, dh, dx: (B, L, D). gate_logits and
+ *          dgate_logits: (B, L, 2D), row (b, t) holding rho in columns [0, D)
+ *          and iota in columns [D, 2D) (the output layout of one Linear layer
+ *          of width 2D). lambda, dlambda: (D). h0, h_last, dh_last, dh0: (B, D).
+ * Dtypes   x, gate_logits, h, dh, dx, dgate_logits use the I/O dtype `io`
+ *          (float32 or bfloat16). lambda, h0, h_last, dh_last, dh0, dlambda and
+ *          the recurrent-step state are always float32. Internal state and all
+ *          arithmetic are float32; bf16 outputs are rounded to nearest-even.
+ * Streams  Every call is asynchronous on `stream` (NULL = the legacy default
+ *          stream) and returns once the work is enqueued.
+ * Checks   Arguments are validated on the host before anything is enqueued:
+ *          a NULL required pointer, a negative size, c <= 0 or not finite, an
+ *          unknown dtype, a too-small workspace or a tensor pointer that is not
+ *          16-byte aligned (4-byte for h0, h_last, dh_last, dh0) returns
+ *          BLR_ERR_INVALID_ARG; D not a multiple of 8, or a problem too large
+ *          for the tiling, returns BLR_ERR_UNSUPPORTED. Nothing is enqueued on
+ *          a validation error. A failed launch returns BLR_ERR_CUDA.
+ * Empty    B == 0 or D == 0 is a no-op. L == 0 is a valid empty sequence:
+ *          h_last = h0 (0 when h0 is NULL); the backward writes dh0 = dh_last
+ *          (0 when NULL) and dlambda = 0.
+ * Domain   Outputs are finite for finite inputs with r_t > 0 and
+ *          softplus(Lambda) > 0 in float32 (|rho| below about 80). At
+ *          alpha_t == 1 exactly the gradient through beta_t is infinite
+ *          (the derivative of sqrt(1 - alpha^2)); such inputs give inf/nan.
+ * Errors   The library never exits, traps or prints. Waits between thread
+ *          blocks are bounded (about one second); an expired wait is recorded
+ *          in the workspace and reported by blr_workspace_status().
+ */
+#ifndef BLR_H_
+#define BLR_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define BLR_API __attribute__((visibility("default")))
+#else
+#define BLR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* blr_stream_t;
+
+typedef enum {
+  BLR_F32 = 0,  /* IEEE binary32 */
+  BLR_BF16 = 1  /* bfloat16 */
+} blr_dtype;
+
+typedef enum {
+  BLR_OK = 0,
+  BLR_ERR_INVALID_ARG = 1,  /* bad pointer, size, alignment, dtype, c or workspace size */
+  BLR_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels handle (D % 8 != 0, too large) */
+  BLR_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed (see blr_last_error_string) */
+  BLR_ERR_TIMEOUT = 4,      /* a bounded wait between thread blocks expired (outputs undefined) */
+  BLR_ERR_WORKSPACE = 5     /* blr_scan_bwd was given a workspace without matching forward carries */
+} blr_status;
+
+/* Problem description of one scan call. */
+typedef struct {
+  int64_t B;    /* batch rows (independent sequences) */
+  int64_t L;    /* sequence length (time steps) */
+  int64_t D;    /* channels (the recurrence is independent per channel) */
+  blr_dtype io; /* dtype of x, gate_logits, h, dh, dx, dgate_logits */
+  float c;      /* decay exponent constant; 1.0 is the paper's alpha = exp(-softplus(Lambda) r) */
+} blr_desc;
+
+/*
+ * Workspace size in bytes for blr_scan_fwd / blr_scan_bwd on `desc`; 0 when
+ * the description is invalid or needs none (B, L or D zero). The workspace
+ * holds per-tile carries of the forward (reused by the backward), per-tile
+ * state of the inter-block scans, and the float64 partial sums of dlambda:
+ * about 24 bytes per channel per tile of up to 64 time steps (under 0.4
+ * bytes per element), plus 64 bytes per channel. It depends only on B, L, D.
+ */
+BLR_API size_t blr_workspace_bytes(const blr_desc* desc);
+
+/*
+ * Forward BD-LRU scan (Sec. 3.2, Eq. linrnn; the scan of Sec. 3.3):
+ *   h[b,t,d] = alpha[b,t,d] * h[b,t-1,d] + beta[b,t,d] * x[b,t,d],
+ *   h[b,-1,d] = h0[b,d]   (h0 == NULL: zero state, as in the paper)
+ * x           (B, L, D)  io dtype, input of the recurrence
+ * gate_logits (B, L, 2D) io dtype, [rho | iota] pre-activations
+ * lambda      (D)        float32, Lambda
+ * h0          (B, D)     float32 or NULL
+ * h           (B, L, D)  io dtype, output; may be NULL to compute only the
+ *                        carries the backward needs (and h_last)
+ * h_last      (B, D)     float32 or NULL, the float32 state h[b, L-1, :]
+ * ws, ws_bytes           device workspace of at least blr_workspace_bytes(desc)
+ *                        bytes, 16-byte aligned. Its previous contents are
+ *                        ignored; on return (in stream order) it holds the
+ *                        per-tile carries that blr_scan_bwd consumes.
+ */
+BLR_API blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_logits,
+                        const float* lambda, const float* h0, void* h, float* h_last, void* ws,
+                        size_t ws_bytes, blr_stream_t stream);
+
+/*
+ * Backward of blr_scan_fwd for the loss  sum_{b,t,d} dh * h + sum_{b,d} dh_last * h_last
+ * (gradients derived from the definitions of Sec. 3.2; the paper prints none).
+ * With g_t = dh_t + alpha_{t+1} g_{t+1} and g_{L-1} = dh_{L-1} + dh_last:
+ *   dx    = g beta                        (direct term only: the gradient through
+ *   drho  = dL/dalpha * dalpha/drho        the caller's gate projections is the
+ *   diota = g sqrt(1-alpha^2) x i (1-i)    caller's, fed by drho and diota)
+ *   dlambda[d] = sum over b, t of the Lambda-derivative (written, not accumulated)
+ *   dh0   = alpha_0 g_0
+ * dh          (B, L, D)  io dtype, upstream gradient of h
+ * dh_last     (B, D)     float32 or NULL (zero)
+ * x, gate_logits, lambda, h0: exactly the forward's inputs
+ * dx          (B, L, D)  io dtype, output
+ * dgate_logits(B, L, 2D) io dtype, output [drho | diota]
+ * dlambda     (D)        float32, output
+ * dh0         (B, D)     float32 or NULL
+ * ws          the workspace a blr_scan_fwd with the same desc and inputs filled
+ *             (h may have been NULL in that call). If ws does not hold
+ *             carries of a completed forward of the same desc, no output is
+ *             written and blr_workspace_status() reports BLR_ERR_WORKSPACE. The
+ *             forward's carries survive the call, so the backward may be repeated.
+ * h_{t-1} is recomputed from the forward's per-tile carries, not read from h.
+ */
+BLR_API blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
+                        const void* gate_logits, const float* lambda, const float* h0, void* dx,
+                        void* dgate_logits, float* dlambda, float* dh0, void* ws, size_t ws_bytes,
+                        blr_stream_t stream);
+
+/*
+ * One recurrent-inference step for a batch of states (the low-cost recurrent
+ * inference of Sec. 1 and Sec. 4.3): h_t = alpha_t * h_prev + beta_t * x_t.
+ * h_prev (B, D) float32; x_t (B, D) io dtype; gate_logits_t (B, 2D) io dtype;
+ * lambda (D) float32; h_t (B, D) float32 output (may alias h_prev exactly).
+ * Needs no workspace.
+ */
+BLR_API blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_prev,
+                    const void* x_t, const void* gate_logits_t, const float* lambda, float* h_t,
+                    blr_stream_t stream);
+
+/*
+ * Synchronises `stream`, then reads the error word that the kernels of
+ * earlier calls on this workspace recorded: BLR_OK, BLR_ERR_TIMEOUT or
+ * BLR_ERR_WORKSPACE (BLR_ERR_CUDA if the read itself fails). The word is
+ * cleared by the next blr_scan_fwd on the workspace.
+ */
+BLR_API blr_status blr_workspace_status(const blr_desc* desc, const void* ws, size_t ws_bytes,
+                                blr_stream_t stream);
+
+/* Static text for a status code. */
+BLR_API const char* blr_status_string(blr_status status);
+
+/* Text of the last BLR_ERR_CUDA / validation failure on the calling host thread. */
+BLR_API const char* blr_last_error_string(void);
+
+/*
+ * Diagnostic: runs one thread block that waits on a workspace flag nothing
+ * sets, with the given bound in nanoseconds (at most 1e9), then records the
+ * expired wait in the workspace. blr_workspace_status() then returns
+ * BLR_ERR_TIMEOUT. This is how the bounded-wait path is tested without a
+ * fault; it touches only the workspace.
+ */
+BLR_API blr_status blr_selftest_wait_timeout(const blr_desc* desc, void* ws, size_t ws_bytes,
+                                     uint64_t timeout_ns, blr_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BLR_H_ */

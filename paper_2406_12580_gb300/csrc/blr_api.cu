@@ -1,0 +1,259 @@
+// C ABI of the BD-LRU scan library (declared in include/blr.h): host-side
+// validation, the tiling plan, workspace clearing and kernel launches. The
+// library allocates nothing and never synchronises except in
+// blr_workspace_status().
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "blr.h"
+#include "blr_kernels.cuh"
+
+namespace {
+
+using blr::Plan;
+
+thread_local char g_last_error[512] = "";
+
+blr_status fail(blr_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+blr_status cuda_check(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return BLR_OK;
+  return fail(BLR_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Shared checks of the problem description; fills `plan` when B, L, D > 0.
+blr_status check_desc(const blr_desc* d, Plan* plan, bool* empty_bd) {
+  if (d == nullptr) return fail(BLR_ERR_INVALID_ARG, "desc is NULL");
+  if (d->B < 0 || d->L < 0 || d->D < 0)
+    return fail(BLR_ERR_INVALID_ARG, "negative size B=%lld L=%lld D=%lld", (long long)d->B,
+                (long long)d->L, (long long)d->D);
+  if (d->io != BLR_F32 && d->io != BLR_BF16)
+    return fail(BLR_ERR_INVALID_ARG, "unknown io dtype %d", (int)d->io);
+  if (!(d->c > 0.0f) || !isfinite(d->c))
+    return fail(BLR_ERR_INVALID_ARG, "c must be finite and > 0");
+  if (d->D % 8 != 0) return fail(BLR_ERR_UNSUPPORTED, "D=%lld is not a multiple of 8", (long long)d->D);
+  *empty_bd = (d->B == 0 || d->D == 0);
+  if (*empty_bd || d->L == 0) return BLR_OK;
+  // Element offsets (b L + t) 2D + d must fit in int64; tile tickets in uint32.
+  if (d->B > (int64_t)1 << 40 || d->L > (int64_t)1 << 40 || d->D > (int64_t)1 << 24 ||
+      (double)d->B * (double)d->L * (double)d->D > 1e18)
+    return fail(BLR_ERR_UNSUPPORTED, "problem too large");
+  blr::make_plan(d->B, d->L, d->D, (int)d->io, d->c, plan);
+  if (plan->n_tiles >= ((int64_t)1 << 31))
+    return fail(BLR_ERR_UNSUPPORTED, "too many tiles (%lld)", (long long)plan->n_tiles);
+  return BLR_OK;
+}
+
+blr_status need(const void* p, const char* name, size_t align) {
+  if (p == nullptr) return fail(BLR_ERR_INVALID_ARG, "%s is NULL", name);
+  if (!aligned(p, align)) return fail(BLR_ERR_INVALID_ARG, "%s is not %zu-byte aligned", name, align);
+  return BLR_OK;
+}
+
+blr_status optional(const void* p, const char* name, size_t align) {
+  if (p != nullptr && !aligned(p, align))
+    return fail(BLR_ERR_INVALID_ARG, "%s is not %zu-byte aligned", name, align);
+  return BLR_OK;
+}
+
+#define BLR_TRY(expr)                  \
+  do {                                 \
+    blr_status s_ = (expr);            \
+    if (s_ != BLR_OK) return s_;       \
+  } while (0)
+
+blr_status check_ws(const Plan& plan, const void* ws, size_t ws_bytes) {
+  BLR_TRY(need(ws, "ws", 16));
+  if (ws_bytes < plan.bytes)
+    return fail(BLR_ERR_INVALID_ARG, "ws_bytes=%zu < required %zu", ws_bytes, plan.bytes);
+  return BLR_OK;
+}
+
+dim3 scan_block(const Plan& p) { return dim3((unsigned)p.nv, (unsigned)p.nt, 1); }
+
+}  // namespace
+
+extern "C" {
+
+size_t blr_workspace_bytes(const blr_desc* desc) {
+  Plan plan;
+  bool empty = false;
+  if (check_desc(desc, &plan, &empty) != BLR_OK || empty || desc->L == 0) return 0;
+  return plan.bytes;
+}
+
+blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_logits,
+                        const float* lambda, const float* h0, void* h, float* h_last, void* ws,
+                        size_t ws_bytes, blr_stream_t stream) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty) return BLR_OK;
+  BLR_TRY(need(lambda, "lambda", 16));
+  BLR_TRY(optional(h0, "h0", 4));
+  BLR_TRY(optional(h_last, "h_last", 4));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const size_t state_bytes = sizeof(float) * (size_t)desc->B * (size_t)desc->D;
+  if (desc->L == 0) {  // empty sequence: the state is unchanged
+    if (h_last == nullptr) return BLR_OK;
+    if (h0 != nullptr)
+      return cuda_check(cudaMemcpyAsync(h_last, h0, state_bytes, cudaMemcpyDeviceToDevice, st),
+                        "copy h0 to h_last");
+    return cuda_check(cudaMemsetAsync(h_last, 0, state_bytes, st), "clear h_last");
+  }
+  BLR_TRY(need(x, "x", 16));
+  BLR_TRY(need(gate_logits, "gate_logits", 16));
+  BLR_TRY(optional(h, "h", 16));
+  BLR_TRY(check_ws(plan, ws, ws_bytes));
+
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  // Clear the forward header (tickets, counters, error word) and tile flags.
+  BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_fhdr, 0, plan.off_bhdr - plan.off_fhdr, st),
+                     "clear forward workspace"));
+  blr::FwdArgs a{plan, x, gate_logits, lambda, h0, h, h_last, w};
+  const dim3 grid((unsigned)plan.n_tiles), block = scan_block(plan);
+  if (desc->io == BLR_F32)
+    blr::scan_fwd_kernel<blr::IoF32, blr::MathPrecise><<<grid, block, 0, st>>>(a);
+  else
+    blr::scan_fwd_kernel<blr::IoBF16, blr::MathFast><<<grid, block, 0, st>>>(a);
+  return cuda_check(cudaGetLastError(), "launch scan_fwd_kernel");
+}
+
+blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
+                        const void* gate_logits, const float* lambda, const float* h0, void* dx,
+                        void* dgate_logits, float* dlambda, float* dh0, void* ws, size_t ws_bytes,
+                        blr_stream_t stream) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty) return BLR_OK;
+  BLR_TRY(need(lambda, "lambda", 16));
+  BLR_TRY(need(dlambda, "dlambda", 4));
+  BLR_TRY(optional(h0, "h0", 4));
+  BLR_TRY(optional(dh_last, "dh_last", 4));
+  BLR_TRY(optional(dh0, "dh0", 4));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (desc->L == 0) {  // empty sequence: dh0 = dh_last, no dependence on Lambda
+    const size_t state_bytes = sizeof(float) * (size_t)desc->B * (size_t)desc->D;
+    BLR_TRY(cuda_check(cudaMemsetAsync(dlambda, 0, sizeof(float) * (size_t)desc->D, st),
+                       "clear dlambda"));
+    if (dh0 == nullptr) return BLR_OK;
+    if (dh_last != nullptr)
+      return cuda_check(cudaMemcpyAsync(dh0, dh_last, state_bytes, cudaMemcpyDeviceToDevice, st),
+                        "copy dh_last to dh0");
+    return cuda_check(cudaMemsetAsync(dh0, 0, state_bytes, st), "clear dh0");
+  }
+  BLR_TRY(need(dh, "dh", 16));
+  BLR_TRY(need(x, "x", 16));
+  BLR_TRY(need(gate_logits, "gate_logits", 16));
+  BLR_TRY(need(dx, "dx", 16));
+  BLR_TRY(need(dgate_logits, "dgate_logits", 16));
+  BLR_TRY(check_ws(plan, ws, ws_bytes));
+
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  // Clear the backward header, the dLambda partial sums and the backward flags.
+  BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_bhdr, 0, plan.off_fagg - plan.off_bhdr, st),
+                     "clear backward workspace"));
+  blr::BwdArgs a{plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda, dh0, w};
+  const dim3 grid((unsigned)plan.n_tiles), block = scan_block(plan);
+  if (desc->io == BLR_F32)
+    blr::scan_bwd_kernel<blr::IoF32, blr::MathPrecise><<<grid, block, 0, st>>>(a);
+  else
+    blr::scan_bwd_kernel<blr::IoBF16, blr::MathFast><<<grid, block, 0, st>>>(a);
+  return cuda_check(cudaGetLastError(), "launch scan_bwd_kernel");
+}
+
+blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_prev,
+                    const void* x_t, const void* gate_logits_t, const float* lambda, float* h_t,
+                    blr_stream_t stream) {
+  if (B < 0 || D < 0) return fail(BLR_ERR_INVALID_ARG, "negative size B=%lld D=%lld", (long long)B, (long long)D);
+  if (io != BLR_F32 && io != BLR_BF16) return fail(BLR_ERR_INVALID_ARG, "unknown io dtype %d", (int)io);
+  if (!(c > 0.0f) || !isfinite(c)) return fail(BLR_ERR_INVALID_ARG, "c must be finite and > 0");
+  if (D % 8 != 0) return fail(BLR_ERR_UNSUPPORTED, "D=%lld is not a multiple of 8", (long long)D);
+  if (B == 0 || D == 0) return BLR_OK;
+  if (D > (int64_t)1 << 24 || B > (int64_t)1 << 40) return fail(BLR_ERR_UNSUPPORTED, "problem too large");
+  BLR_TRY(need(h_prev, "h_prev", 16));
+  BLR_TRY(need(x_t, "x_t", 16));
+  BLR_TRY(need(gate_logits_t, "gate_logits_t", 16));
+  BLR_TRY(need(lambda, "lambda", 16));
+  BLR_TRY(need(h_t, "h_t", 16));
+  constexpr int kRows = 4;
+  const int vec = (io == BLR_F32) ? blr::IoF32::kVec : blr::IoBF16::kVec;
+  const int64_t nvec = D / vec;
+  const int bx = (int)(nvec < 64 ? nvec : 64);
+  const int by = 256 / bx;
+  const int64_t n_vgroups = (nvec + bx - 1) / bx;
+  const int64_t rows_per_block = (int64_t)by * kRows;
+  const int64_t n_rgroups = (B + rows_per_block - 1) / rows_per_block;
+  if (n_vgroups * n_rgroups >= ((int64_t)1 << 31)) return fail(BLR_ERR_UNSUPPORTED, "grid too large");
+  blr::StepArgs a{B, D, c, kRows, n_vgroups, h_prev, x_t, gate_logits_t, lambda, h_t};
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const dim3 grid((unsigned)(n_vgroups * n_rgroups)), block((unsigned)bx, (unsigned)by);
+  if (io == BLR_F32)
+    blr::step_kernel<blr::IoF32, blr::MathPrecise, kRows><<<grid, block, 0, st>>>(a);
+  else
+    blr::step_kernel<blr::IoBF16, blr::MathFast, kRows><<<grid, block, 0, st>>>(a);
+  return cuda_check(cudaGetLastError(), "launch step_kernel");
+}
+
+blr_status blr_workspace_status(const blr_desc* desc, const void* ws, size_t ws_bytes,
+                                blr_stream_t stream) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty || desc->L == 0) return BLR_OK;
+  BLR_TRY(check_ws(plan, ws, ws_bytes));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t err = 0;
+  const unsigned char* w = static_cast<const unsigned char*>(ws);
+  BLR_TRY(cuda_check(cudaMemcpyAsync(&err, w + plan.off_fhdr + offsetof(blr::FwdHeader, err),
+                                     sizeof(err), cudaMemcpyDeviceToHost, st),
+                     "read workspace error word"));
+  BLR_TRY(cuda_check(cudaStreamSynchronize(st), "synchronize stream"));
+  if (err & blr::kErrTimeout) return BLR_ERR_TIMEOUT;
+  if (err & blr::kErrWorkspace) return BLR_ERR_WORKSPACE;
+  return BLR_OK;
+}
+
+blr_status blr_selftest_wait_timeout(const blr_desc* desc, void* ws, size_t ws_bytes,
+                                     uint64_t timeout_ns, blr_stream_t stream) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty || desc->L == 0) return fail(BLR_ERR_INVALID_ARG, "the self-test needs a non-empty problem");
+  BLR_TRY(check_ws(plan, ws, ws_bytes));
+  if (timeout_ns > blr::kWaitTimeoutNs) return fail(BLR_ERR_INVALID_ARG, "timeout_ns above 1e9");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  uint32_t* flag = reinterpret_cast<uint32_t*>(w + plan.off_bhdr + offsetof(blr::BwdHeader, selftest_flag));
+  uint32_t* err = reinterpret_cast<uint32_t*>(w + plan.off_fhdr + offsetof(blr::FwdHeader, err));
+  BLR_TRY(cuda_check(cudaMemsetAsync(flag, 0, sizeof(uint32_t), st), "clear self-test flag"));
+  blr::selftest_wait_kernel<<<1, 32, 0, st>>>(flag, err, timeout_ns);
+  return cuda_check(cudaGetLastError(), "launch selftest_wait_kernel");
+}
+
+const char* blr_status_string(blr_status status) {
+  switch (status) {
+    case BLR_OK: return "BLR_OK";
+    case BLR_ERR_INVALID_ARG: return "BLR_ERR_INVALID_ARG: invalid argument";
+    case BLR_ERR_UNSUPPORTED: return "BLR_ERR_UNSUPPORTED: unsupported problem";
+    case BLR_ERR_CUDA: return "BLR_ERR_CUDA: CUDA error";
+    case BLR_ERR_TIMEOUT: return "BLR_ERR_TIMEOUT: a bounded inter-block wait expired";
+    case BLR_ERR_WORKSPACE: return "BLR_ERR_WORKSPACE: workspace holds no matching forward carries";
+  }
+  return "unknown blr_status";
+}
+
+const char* blr_last_error_string(void) { return g_last_error; }
+
+}  // extern "C"

@@ -1,0 +1,246 @@
+"""GPU: the CUDA path (through the C ABI) against the float64 oracle.
+
+Every comparison uses the same seeded inputs on both sides (bf16 inputs are
+rounded once by the generator; the oracle upcasts them). Errors are normwise:
+max|gpu - oracle| / max|oracle| <= 1e-5 for float32 I/O and <= 2e-2 for
+bfloat16 I/O.
+"""
+import numpy as np
+import pytest
+
+from gpu_common import (TOL, compare, gpu_outputs, gpu_scan, gpu_step, normwise, oracle_outputs)
+from paper_2406_12580_gb300 import inputs as I
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # collected on CPU machines, but never run there
+    pytest.skip("no CUDA device", allow_module_level=True)
+
+# Small and ragged shapes the oracle runs in full: a single element, one and
+# several partial tiles, a partial channel block (D = 72 = 64 + 8), the
+# minimal channel width, long look-back chains, slow decays, random h0 and
+# dh_last, and c != 1.
+SMALL = [
+    dict(B=1, L=1, D=8),
+    dict(B=2, L=3, D=8, random_h0=True, random_dh_last=True),
+    dict(B=3, L=7, D=16),
+    dict(B=4, L=50, D=64),
+    dict(B=3, L=65, D=72, random_h0=True, random_dh_last=True),
+    dict(B=2, L=300, D=16, random_h0=True),
+    dict(B=1, L=4000, D=8, random_dh_last=True),
+    dict(B=2, L=1031, D=256, decay=(0.99, 0.9999), random_h0=True, random_dh_last=True),
+    dict(B=5, L=129, D=128, c=2.5, random_h0=True),
+    dict(B=2, L=200, D=64, gate_std=3.0, x_std=4.0),
+]
+
+
+def _cfg(io, seed, **kw):
+    return I.ScanConfig(f"small {kw} {io}", io=io, seed=seed, **kw)
+
+
+@pytest.mark.parametrize("io", [I.F32, I.BF16])
+@pytest.mark.parametrize("case", range(len(SMALL)))
+def test_small_shapes(io, case):
+    inp = I.make_scan_inputs(_cfg(io, 100 + case, **SMALL[case]))
+    buf = gpu_scan(inp)
+    compare(inp, gpu_outputs(buf), oracle_outputs(inp))
+
+
+@pytest.mark.parametrize("k", [0, 1, 2])
+def test_config_full_oracle(k):
+    """Configurations 0-2 at full size against the full oracle."""
+    inp = I.make_scan_inputs(I.CONFIGS[k])
+    buf = gpu_scan(inp)
+    errs = compare(inp, gpu_outputs(buf), oracle_outputs(inp, threads=0))
+    print(f"config {k}: {errs}")
+
+
+def _sampled_channels(D):
+    return sorted({0, 1, 7, 8, 63, 64, 65, D // 2, D - 9, D - 1} & set(range(D)))
+
+
+@pytest.mark.parametrize("k", [3, 4])
+def test_config_full_size_sampled(k):
+    """Configurations 3-4 at full size; the oracle runs the sampled channels in
+    full (every batch row and step of each: the recurrence is per channel)."""
+    inp = I.make_scan_inputs(I.CONFIGS[k])
+    buf = gpu_scan(inp)
+    dsel = _sampled_channels(inp.cfg.D)
+    errs = compare(inp, gpu_outputs(buf, dsel), oracle_outputs(inp, dsel, threads=0))
+    print(f"config {k}: {errs}")
+
+
+@pytest.mark.parametrize("io", [I.F32, I.BF16])
+def test_step_full(io):
+    cfg = I.StepConfig(f"step {io}", B=65536, D=64, io=io, seed=4)
+    s = I.make_step_inputs(cfg)
+    buf = gpu_step(s)
+    import oracle
+    want = oracle.load().step(s.h_prev, s.x, s.gl, s.lam, c=cfg.c)
+    got = buf.h_t.cpu().numpy().astype(np.float64)
+    # the state is float32 in both dtypes; bf16 only rounds the inputs, which
+    # both sides share, and the fast gate arithmetic stays near 1e-6
+    assert normwise(got, want) <= (1e-5 if io == I.F32 else 1e-4)
+
+
+def test_step_small_and_aliased():
+    cfg = I.StepConfig("step small", B=3, D=24, io=I.F32, seed=9)
+    s = I.make_step_inputs(cfg)
+    import oracle
+    want = oracle.load().step(s.h_prev, s.x, s.gl, s.lam)
+    from paper_2406_12580_gb300 import BLR_F32, blr_step
+    from paper_2406_12580_gb300.device import to_device
+    h = to_device(s.h_prev, "f32", "cuda")
+    x = to_device(s.x, "f32", "cuda")
+    gl = to_device(s.gl, "f32", "cuda")
+    lam = to_device(s.lam, "f32", "cuda")
+    blr_step(3, 24, BLR_F32, 1.0, h, x, gl, lam, h)  # in place: h_t aliases h_prev
+    torch.cuda.synchronize()
+    assert normwise(h.cpu().numpy(), want) <= 1e-5
+
+
+def test_padding_rows_are_exact_zeros():
+    """Config 2's left-padded rows (x = rho = iota = 0, h0 = 0) stay exactly 0
+    (the embedding-padding claim of Sec. 3.3), and diota vanishes there."""
+    inp = I.make_scan_inputs(I.scaled(I.CONFIGS[2], B=256))
+    buf = gpu_scan(inp)
+    p = inp.cfg.pad_rows
+    assert torch.count_nonzero(buf.h[:, :p]).item() == 0
+    assert torch.count_nonzero(buf.dgl[:, :p, inp.cfg.D:]).item() == 0
+    # and the real rows equal a run without the padding
+    cfg2 = I.scaled(inp.cfg, L=inp.cfg.L - p, pad_frac=0.0)
+    inp2 = I.make_scan_inputs(cfg2)
+    inp2.x, inp2.gl = inp.x[:, p:].copy(), inp.gl[:, p:].copy()
+    inp2.bits = {k: np.ascontiguousarray(v[:, p:]) for k, v in inp.bits.items()}
+    inp2.dh = inp.dh[:, p:].copy()
+    buf2 = gpu_scan(inp2, with_bwd=False)
+    # chunk boundaries move with the padding, so float32 rounding may differ
+    assert normwise(buf.h[:, p:].float().cpu().numpy(), buf2.h.float().cpu().numpy()) <= 1e-2
+
+
+def test_split_resume():
+    cfg = I.ScanConfig("split", B=3, L=500, D=64, io=I.F32, seed=31, random_h0=True)
+    inp = I.make_scan_inputs(cfg)
+    full = gpu_scan(inp, with_bwd=False)
+    k = 217
+    a = I.make_scan_inputs(I.scaled(cfg, L=k))
+    a.x, a.gl, a.h0 = inp.x[:, :k].copy(), inp.gl[:, :k].copy(), inp.h0
+    ba = gpu_scan(a, with_bwd=False)
+    b = I.make_scan_inputs(I.scaled(cfg, L=cfg.L - k))
+    b.x, b.gl, b.h0 = inp.x[:, k:].copy(), inp.gl[:, k:].copy(), ba.h_last.cpu().numpy()
+    bb = gpu_scan(b, with_bwd=False)
+    got = torch.cat([ba.h, bb.h], dim=1).cpu().numpy()
+    assert normwise(got, full.h.cpu().numpy()) <= 1e-6
+    assert normwise(bb.h_last.cpu().numpy(), full.h_last.cpu().numpy()) <= 1e-6
+
+
+def test_carries_only_forward_then_backward():
+    cfg = I.ScanConfig("carries", B=4, L=700, D=64, io=I.F32, seed=32, random_h0=True,
+                       random_dh_last=True)
+    inp = I.make_scan_inputs(cfg)
+    from paper_2406_12580_gb300.device import ScanBuffers
+    buf = ScanBuffers.from_inputs(inp)
+    buf.h.fill_(7.0)
+    buf.fwd(write_h=False)
+    buf.bwd()
+    torch.cuda.synchronize()
+    assert torch.all(buf.h == 7.0)  # h untouched
+    want = oracle_outputs(inp)
+    got = gpu_outputs(buf)
+    for k in ("h_last", "dx", "dgl", "dlam", "dh0"):
+        assert normwise(got[k], want[k]) <= TOL[I.F32], k
+    # the backward can be repeated on the same workspace
+    buf.bwd()
+    torch.cuda.synchronize()
+    got2 = gpu_outputs(buf)
+    for k in ("dx", "dgl", "dlam", "dh0"):
+        assert normwise(got2[k], want[k]) <= TOL[I.F32], k
+
+
+def test_empty_sequence_and_batch():
+    from paper_2406_12580_gb300 import Desc, blr_scan_bwd, blr_scan_fwd
+    B, D = 3, 16
+    h0 = torch.randn(B, D, device="cuda")
+    dh_last = torch.randn(B, D, device="cuda")
+    lam = torch.randn(D, device="cuda")
+    h_last = torch.full((B, D), 5.0, device="cuda")
+    e = torch.empty(0, device="cuda")
+    blr_scan_fwd(Desc(B, 0, D), e, e, lam, h0, e, h_last, None)
+    dlam = torch.full((D,), 5.0, device="cuda")
+    dh0 = torch.full((B, D), 5.0, device="cuda")
+    blr_scan_bwd(Desc(B, 0, D), e, dh_last, e, e, lam, h0, e, e, dlam, dh0, None)
+    torch.cuda.synchronize()
+    assert torch.equal(h_last, h0) and torch.equal(dh0, dh_last)
+    assert torch.count_nonzero(dlam).item() == 0
+    blr_scan_fwd(Desc(B, 0, D), e, e, lam, None, e, h_last, None)
+    blr_scan_bwd(Desc(B, 0, D), e, None, e, e, lam, None, e, e, dlam, dh0, None)
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(h_last).item() == 0 and torch.count_nonzero(dh0).item() == 0
+    blr_scan_fwd(Desc(0, 10, D), e, e, lam, None, e, None, None)  # B = 0: nothing to do
+
+
+def test_backward_without_forward_carries_is_reported():
+    from paper_2406_12580_gb300 import (BLR_ERR_WORKSPACE, BLR_OK, Desc, blr_workspace_status)
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = I.ScanConfig("ws", B=2, L=300, D=64, io=I.F32, seed=33)
+    inp = I.make_scan_inputs(cfg)
+    buf = ScanBuffers.from_inputs(inp)
+    buf.ws.zero_()
+    buf.dx.fill_(3.0)
+    buf.bwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_ERR_WORKSPACE
+    assert torch.all(buf.dx == 3.0)
+    buf.fwd()  # a forward clears the error word and fills the carries
+    buf.bwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_OK
+    # a forward of another length leaves carries that do not match this problem
+    other = Desc(2, 299, 64)
+    from paper_2406_12580_gb300 import blr_scan_fwd
+    blr_scan_fwd(other, buf.x, buf.gl, buf.lam, None, None, None, buf.ws)
+    buf.bwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_ERR_WORKSPACE
+
+
+def test_bounded_wait_reports_timeout():
+    from paper_2406_12580_gb300 import (BLR_ERR_TIMEOUT, BLR_OK, blr_selftest_wait_timeout,
+                                        blr_workspace_status)
+    from paper_2406_12580_gb300.device import ScanBuffers
+    inp = I.make_scan_inputs(I.ScanConfig("timeout", B=2, L=100, D=64, io=I.F32, seed=34))
+    buf = ScanBuffers.from_inputs(inp)
+    buf.fwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_OK
+    blr_selftest_wait_timeout(buf.desc, buf.ws, 20_000_000)  # 20 ms on a flag nothing sets
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_ERR_TIMEOUT
+    buf.fwd()  # the context is still usable and the next forward clears the word
+    buf.bwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_OK
+    compare(inp, gpu_outputs(buf), oracle_outputs(inp))
+
+
+def test_autograd_wrapper():
+    from paper_2406_12580_gb300 import BDLRUScan
+    cfg = I.ScanConfig("autograd", B=3, L=90, D=32, io=I.F32, seed=35, random_h0=True,
+                       random_dh_last=True)
+    inp = I.make_scan_inputs(cfg)
+    dev = "cuda"
+    x = torch.tensor(inp.x, device=dev, requires_grad=True)
+    gl = torch.tensor(inp.gl, device=dev, requires_grad=True)
+    lam = torch.tensor(inp.lam, device=dev, requires_grad=True)
+    h0 = torch.tensor(inp.h0, device=dev, requires_grad=True)
+    h, h_last = BDLRUScan.apply(x, gl, lam, h0, 1.0)
+    loss = (h * torch.tensor(inp.dh, device=dev)).sum() + (h_last * torch.tensor(inp.dh_last, device=dev)).sum()
+    loss.backward()
+    want = oracle_outputs(inp)
+    assert normwise(h.detach().cpu().numpy(), want["h"]) <= 1e-5
+    assert normwise(x.grad.cpu().numpy(), want["dx"]) <= 1e-5
+    assert normwise(gl.grad.cpu().numpy(), want["dgl"]) <= 1e-5
+    assert normwise(lam.grad.cpu().numpy(), want["dlam"]) <= 1e-5
+    assert normwise(h0.grad.cpu().numpy(), want["dh0"]) <= 1e-5
+
+
+def test_binding_rejects_host_tensors():
+    from paper_2406_12580_gb300 import Desc, blr_scan_fwd
+    x = torch.zeros(1, 4, 8)
+    with pytest.raises(ValueError):
+        blr_scan_fwd(Desc(1, 4, 8), x, x, x, None, x, None, x)
