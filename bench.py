@@ -1,0 +1,498 @@
+#!/usr/bin/env python
+"""Benchmark of the GB300 BD-LRU scan (RecBLR, arXiv 2406.12580, Sec. 3.2-3.3).
+
+One step = one forward scan plus one backward scan (the whole training hot
+path: gates, decay and input normalisation, forward scan, reverse scan,
+dLambda) over one batch of synthetic input, the B=256, L=200, D=64 float32
+workload (ML-1M's maximum length and the paper's embedding width). Inputs are
+resident in HBM when the timed region starts; L2 is flushed (a 2x L2 write)
+before every timed step; each step is timed on the device with CUDA events.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line on rank 0. Under torchrun each rank runs its own replica
+of the workload (the scan shards over batch rows and channels with no
+exchange), so the value is the sum over ranks ("weak" scaling).
+
+--impl reference times the float64 CPU oracle, as it stands, on the host
+cores (there is no other implementation of this method to compare against).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "BD-LRU scan fwd+bwd elements/s and achieved HBM GB/s vs GB300 peak (1 GPU)"
+UNIT = "elements/s"
+FALLBACK_HBM_GBS = 6800.0
+
+# Compulsory HBM bytes per element (inputs read once, outputs written once;
+# the per-tile carries and O(B*D) state are overhead, not counted):
+#   forward : x, rho, iota read, h written             = 4 values
+#   backward: dh, x, rho, iota read, dx, drho, diota   = 7 values
+#   step    : h_prev (f32), x, rho, iota read, h_t (f32) written
+FWD_VALUES, BWD_VALUES = 4, 7
+
+
+def io_bytes(io: str) -> int:
+    return 2 if io == "bf16" else 4
+
+
+def step_bytes_per_elem(io: str) -> int:
+    return 4 + 3 * io_bytes(io) + 4
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=1, help="workload (0-4); 1 is the headline")
+    ap.add_argument("--quick", action="store_true", help="skip the other workloads and e2e")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_sources_sha() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2406_12580_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except Exception:
+        return None
+    if d.get("sources_sha") != kernel_sources_sha():
+        return None
+    return d.get("kernels", {}).get(kernel, {}).get(workload)
+
+
+# ------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+
+    QUERY = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.t0 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t0 = time.time()
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return []
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=10)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            if self.uuid and self.uuid not in f[0]:
+                continue
+            try:
+                rows.append(dict(sm=float(f[1]), sm_max=float(f[2]), power=float(f[3]),
+                                 hw_slowdown=f[5] == "Active", hw_thermal=f[6] == "Active",
+                                 sw_thermal=f[7] == "Active", sw_power_cap=f[8] == "Active"))
+            except ValueError:
+                continue
+        return rows
+
+    @staticmethod
+    def summary(rows):
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        loaded = [r for r in rows if r["power"] > 200.0] or rows
+        reasons = sorted({k for r in loaded for k in ("hw_slowdown", "hw_thermal", "sw_thermal",
+                                                      "sw_power_cap") if r[k]})
+        return {"sm_mhz": statistics.median(r["sm"] for r in loaded),
+                "sm_max_mhz": max(r["sm_max"] for r in rows), "reasons": reasons,
+                "samples": len(loaded), "power_w_max": max(r["power"] for r in rows)}
+
+
+# ------------------------------------------------------------ CPU baseline
+
+def cpu_oracle_rate(inp, target_s: float = 10.0, max_reps: int = 50):
+    """The float64 oracle, as it stands, on the host cores: fwd + bwd over the
+    whole workload, repeated for about `target_s` seconds. Returns
+    (elements/s, threads, reps, seconds)."""
+    import oracle
+    orc = oracle.load()
+    threads = os.cpu_count() or 1
+    n = inp.cfg.elements
+    t = time.perf_counter()
+    reps = 0
+    while True:
+        orc.fwd(inp.x, inp.gl, inp.lam, inp.h0, c=inp.cfg.c, threads=threads)
+        if inp.dh is not None:
+            orc.bwd(inp.dh, inp.x, inp.gl, inp.lam, inp.h0, inp.dh_last, c=inp.cfg.c,
+                    threads=threads)
+        reps += 1
+        el = time.perf_counter() - t
+        if el >= target_s or reps >= max_reps:
+            break
+    threads_used = threads if orc.has_openmp else 1
+    return n * reps / el, threads_used, reps, el
+
+
+# --------------------------------------------------------------- reference
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2406_12580_gb300 import inputs as I
+    import oracle
+    orc = oracle.load()
+    cfg = I.CONFIGS[args.config]
+    threads = os.cpu_count() or 1
+    # One reference step = fwd + bwd of the oracle over a bounded sample of the
+    # workload (whole batch rows), sized to about one second.
+    probe = I.make_scan_inputs(I.scaled(cfg, B=max(1, min(cfg.B, 8))))
+    t = time.perf_counter()
+    orc.fwd(probe.x, probe.gl, probe.lam, probe.h0, threads=threads)
+    if probe.dh is not None:
+        orc.bwd(probe.dh, probe.x, probe.gl, probe.lam, probe.h0, probe.dh_last, threads=threads)
+    per_row = (time.perf_counter() - t) / probe.cfg.B
+    Bs = int(max(1, min(cfg.B, 1.0 / max(per_row, 1e-9))))
+    inp = I.make_scan_inputs(I.scaled(cfg, B=Bs))
+
+    def step():
+        orc.fwd(inp.x, inp.gl, inp.lam, inp.h0, threads=threads)
+        if inp.dh is not None:
+            orc.bwd(inp.dh, inp.x, inp.gl, inp.lam, inp.h0, inp.dh_last, threads=threads)
+
+    for _ in range(args.warmup):
+        step()
+    t = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t
+    value = inp.cfg.elements * args.steps / el
+    sample = f"{Bs} of {cfg.B} batch rows of {cfg.name} per step (fwd+bwd, float64 oracle)"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads if orc.has_openmp else 1,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# -------------------------------------------------------------------- ours
+
+def time_scan(buf, reps, flush, with_bwd=True):
+    """Per-rep device time (ms) of the forward and the backward, L2 flushed
+    before each rep."""
+    import torch
+    fwd_ms, bwd_ms = [], []
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    for k in range(reps):
+        flush()
+        e0, e1, e2 = ev[k]
+        e0.record()
+        buf.fwd()
+        e1.record()
+        if with_bwd:
+            buf.bwd()
+        e2.record()
+    torch.cuda.synchronize()
+    for e0, e1, e2 in ev:
+        fwd_ms.append(e0.elapsed_time(e1))
+        bwd_ms.append(e1.elapsed_time(e2))
+    return fwd_ms, bwd_ms
+
+
+def time_step_kernel(sbuf, reps, flush):
+    import torch
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps)]
+    for k in range(reps):
+        flush()
+        ev[k][0].record()
+        sbuf.step()
+        ev[k][1].record()
+    torch.cuda.synchronize()
+    return [a.elapsed_time(b) for a, b in ev]
+
+
+def workload_summary(cfg, fwd_ms, bwd_ms, peak):
+    n = cfg.elements
+    f = statistics.median(fwd_ms)
+    b = statistics.median(bwd_ms) if bwd_ms else 0.0
+    ib = io_bytes(cfg.io)
+    out = {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io,
+           "fwd_ms": f, "fwd_gbs": n * FWD_VALUES * ib / (f * 1e-3) / 1e9}
+    out["fwd_frac"] = out["fwd_gbs"] / peak
+    if not cfg.fwd_only:
+        out.update(bwd_ms=b, bwd_gbs=n * BWD_VALUES * ib / (b * 1e-3) / 1e9)
+        out["bwd_frac"] = out["bwd_gbs"] / peak
+        out["elements_per_s"] = n / ((f + b) * 1e-3)
+        out["fwd_bwd_gbs"] = n * (FWD_VALUES + BWD_VALUES) * ib / ((f + b) * 1e-3) / 1e9
+        out["fwd_bwd_frac"] = out["fwd_bwd_gbs"] / peak
+    else:
+        out["elements_per_s"] = n / (f * 1e-3)
+    return out
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import ScanBuffers, StepBuffers, to_device
+
+    peak, peak_kind = measured_peaks()
+    props = torch.cuda.get_device_properties(dev)
+    l2 = int(getattr(props, "L2_cache_size", 126 * 2**20) or 126 * 2**20)
+    flush_buf = torch.empty(2 * l2 // 4 + 1024, dtype=torch.float32, device=dev)
+    flush = lambda: flush_buf.fill_(1.0)  # noqa: E731
+
+    cfg = I.CONFIGS[args.config]
+    inp = I.make_scan_inputs(cfg)
+    buf = ScanBuffers.from_inputs(inp, device=dev)
+    n = cfg.elements
+
+    def step():
+        buf.fwd()
+        if not cfg.fwd_only:
+            buf.bwd()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    uuid = None
+    try:
+        uuid = str(props.uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    # Untimed pre-roll of the same steps (about 0.5 s) so that the clock
+    # samples see the GPU under this load before and during the timed region.
+    t_pre = time.time()
+    preroll = 0
+    while time.time() - t_pre < 0.5:
+        for _ in range(20):
+            flush()
+            step()
+        preroll += 20
+        torch.cuda.synchronize()
+
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    fwd_ms, bwd_ms = time_scan(buf, args.steps, flush, with_bwd=not cfg.fwd_only)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    wall = time.perf_counter() - wall0
+    clock_rows = sampler.stop()
+
+    total_ms = sum(fwd_ms) + sum(bwd_ms)
+    t_local = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        torch.distributed.all_reduce(t_local, op=torch.distributed.ReduceOp.MAX)
+    t_max_ms = float(t_local.item())
+    value = world * n * args.steps / (t_max_ms * 1e-3)
+    summ = workload_summary(cfg, fwd_ms, bwd_ms, peak)
+
+    # dominant kernel of the step and its roofline
+    favg = sum(fwd_ms) / len(fwd_ms)
+    bavg = sum(bwd_ms) / len(bwd_ms) if bwd_ms and not cfg.fwd_only else 0.0
+    ib = io_bytes(cfg.io)
+    if bavg > favg:
+        kname, avg_ms, alg = "scan_bwd_kernel", bavg, n * BWD_VALUES * ib
+    else:
+        kname, avg_ms, alg = "scan_fwd_kernel", favg, n * FWD_VALUES * ib
+    achieved = alg / (avg_ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
+                "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": ncu_traffic(kname, f"config{args.config}"),
+                "algorithmic_bytes_per_launch": alg,
+                "timing": "CUDA events around each C-ABI call (kernel plus its workspace clear)"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": max(3, args.warmup), "preroll_steps": preroll,
+        "ms_per_step": t_max_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32" if cfg.io == "f32" else "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io,
+                   "state": "f32", "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "l2": f"flushed before every timed step ({2 * l2 >> 20} MiB write)",
+                   "inputs": "seeded synthetic (paper_2406_12580_gb300.inputs), resident in HBM"},
+        "hbm_gbs": summ.get("fwd_bwd_gbs", summ["fwd_gbs"]),
+        "hbm_frac": summ.get("fwd_bwd_frac", summ["fwd_frac"]),
+        "roofline": roofline,
+        "gpu_launches": (1 if cfg.fwd_only else 2) * args.steps,
+        "wall_s_timed_region": wall,
+        "per_kernel": summ,
+    }
+
+    rows_summary = ClockSampler.summary(clock_rows)
+    line["clocks"] = {k: rows_summary[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")}
+    line["clocks"]["samples"] = rows_summary["samples"]
+    line["clocks"]["window"] = "0.5 s pre-roll of the same steps plus the timed region"
+
+    if rank == 0 and not args.quick:
+        # end to end through the public API: pinned host inputs -> HBM, fwd,
+        # bwd, results -> pinned host, every step
+        line["e2e"] = e2e(buf, inp, min(args.steps, 20), world)
+        line["other_workloads"] = other_workloads(flush, peak, dev, args.config)
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, threads, reps, secs = cpu_oracle_rate(inp)
+        line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+                                "sample": f"{reps} x fwd+bwd of the whole workload "
+                                          f"({n} elements) in {secs:.1f} s, float64"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def e2e(buf, inp, reps, world):
+    """Same metric through the C ABI with host buffers: every step copies the
+    inputs from pinned host memory and reads every output back."""
+    import torch
+    from paper_2406_12580_gb300.device import to_device
+    cfg = inp.cfg
+    pin = lambda name: to_device(inp.io_array(name), cfg.io, "cpu", pin=False).pin_memory()  # noqa: E731
+    hx, hgl, hdh = pin("x"), pin("gl"), pin("dh") if not cfg.fwd_only else None
+    outs = [buf.h, buf.h_last] + ([] if cfg.fwd_only else [buf.dx, buf.dgl, buf.dlam])
+    host_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    h2d = sum(t.numel() * t.element_size() for t in (hx, hgl, hdh) if t is not None)
+    d2h = sum(t.numel() * t.element_size() for t in host_outs)
+    times = []
+    for k in range(reps + 3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        buf.x.copy_(hx, non_blocking=True)
+        buf.gl.copy_(hgl, non_blocking=True)
+        if hdh is not None:
+            buf.dh.copy_(hdh, non_blocking=True)
+        buf.fwd()
+        if not cfg.fwd_only:
+            buf.bwd()
+        for d, s in zip(host_outs, outs):
+            d.copy_(s, non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize()
+        if k >= 3:
+            times.append(e0.elapsed_time(e1))
+    ms = statistics.median(times)
+    return {"value": world * cfg.elements / (ms * 1e-3), "unit": UNIT, "ms_per_step": ms,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+
+def other_workloads(flush, peak, dev, headline):
+    """The other benchmark workloads (fewer repetitions; the same timing)."""
+    import torch
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import ScanBuffers, StepBuffers
+    out = {}
+    for k in (0, 1, 2, 3, 4):
+        if k == headline:
+            continue
+        cfg = I.CONFIGS[k]
+        inp = I.make_scan_inputs(cfg)
+        buf = ScanBuffers.from_inputs(inp, device=dev)
+        time_scan(buf, 3, flush, with_bwd=not cfg.fwd_only)
+        f, b = time_scan(buf, 10, flush, with_bwd=not cfg.fwd_only)
+        out[f"config{k}"] = workload_summary(cfg, f, b, peak)
+        del buf, inp
+        torch.cuda.empty_cache()
+    for io in ("f32", "bf16"):
+        scfg = I.StepConfig(f"recurrent step B=65536 D=64 {io}", 65536, 64, io, seed=4)
+        sbuf = StepBuffers.from_inputs(I.make_step_inputs(scfg), device=dev)
+        time_step_kernel(sbuf, 3, flush)
+        ms = statistics.median(time_step_kernel(sbuf, 20, flush))
+        gbs = scfg.elements * step_bytes_per_elem(io) / (ms * 1e-3) / 1e9
+        out[f"step_{io}"] = {"workload": scfg.name, "ms": ms,
+                             "elements_per_s": scfg.elements / (ms * 1e-3), "gbs": gbs,
+                             "frac": gbs / peak}
+    return out
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

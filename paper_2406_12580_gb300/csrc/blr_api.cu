@@ -44,13 +44,13 @@ blr_status check_desc(const blr_desc* d, Plan* plan, bool* empty_bd) {
   if (d->D % 8 != 0) return fail(BLR_ERR_UNSUPPORTED, "D=%lld is not a multiple of 8", (long long)d->D);
   *empty_bd = (d->B == 0 || d->D == 0);
   if (*empty_bd || d->L == 0) return BLR_OK;
-  // Element offsets (b L + t) 2D + d must fit in int64; tile tickets in uint32.
+  // Element offsets (b L + t) 2D + d must fit in int64; tile tickets in int32.
   if (d->B > (int64_t)1 << 40 || d->L > (int64_t)1 << 40 || d->D > (int64_t)1 << 24 ||
       (double)d->B * (double)d->L * (double)d->D > 1e18)
     return fail(BLR_ERR_UNSUPPORTED, "problem too large");
   blr::make_plan(d->B, d->L, d->D, (int)d->io, d->c, plan);
-  if (plan->n_tiles >= ((int64_t)1 << 31))
-    return fail(BLR_ERR_UNSUPPORTED, "too many tiles (%lld)", (long long)plan->n_tiles);
+  if (plan->n_tiles_f >= ((int64_t)1 << 30) || plan->n_tiles_b >= ((int64_t)1 << 30))
+    return fail(BLR_ERR_UNSUPPORTED, "too many tiles (%lld)", (long long)plan->n_tiles_b);
   return BLR_OK;
 }
 
@@ -79,7 +79,38 @@ blr_status check_ws(const Plan& plan, const void* ws, size_t ws_bytes) {
   return BLR_OK;
 }
 
-dim3 scan_block(const Plan& p) { return dim3((unsigned)p.nv, (unsigned)p.nt, 1); }
+// Persistent grid: as many blocks as fit on the device at once, at most one
+// per tile.
+template <typename K>
+blr_status persistent_grid(K kernel, int threads, int64_t n_tiles, unsigned* grid) {
+  int dev = 0, sms = 0, per_sm = 0;
+  BLR_TRY(cuda_check(cudaGetDevice(&dev), "cudaGetDevice"));
+  BLR_TRY(cuda_check(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev),
+                     "query SM count"));
+  BLR_TRY(cuda_check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0),
+                     "query occupancy"));
+  int64_t g = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+  if (g > n_tiles) g = n_tiles;
+  *grid = (unsigned)(g > 0 ? g : 1);
+  return BLR_OK;
+}
+
+// Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
+// empty record pattern and writes k = -c softplus(Lambda).
+blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fill,
+                       size_t fill_bytes, float* k, const float* lambda, int64_t D, float c,
+                       cudaStream_t st) {
+  const int64_t words = (int64_t)(zero_bytes / 4);
+  const int64_t vec4 = (int64_t)(fill_bytes / 16);
+  int64_t work = words > D ? words : D;
+  if (vec4 > work) work = vec4;
+  int64_t blocks = (work + 255) / 256;
+  if (blocks > 2048) blocks = 2048;
+  blr::prep_kernel<<<(unsigned)blocks, 256, 0, st>>>(reinterpret_cast<uint32_t*>(zero), words,
+                                                     reinterpret_cast<uint4*>(fill), vec4, k,
+                                                     lambda, D, c);
+  return cuda_check(cudaGetLastError(), "launch prep_kernel");
+}
 
 }  // namespace
 
@@ -117,15 +148,23 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
-  // Clear the forward header (tickets, counters, error word) and tile flags.
-  BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_fhdr, 0, plan.off_bhdr - plan.off_fhdr, st),
-                     "clear forward workspace"));
-  blr::FwdArgs a{plan, x, gate_logits, lambda, h0, h, h_last, w};
-  const dim3 grid((unsigned)plan.n_tiles), block = scan_block(plan);
-  if (desc->io == BLR_F32)
-    blr::scan_fwd_kernel<blr::IoF32, blr::MathPrecise><<<grid, block, 0, st>>>(a);
-  else
-    blr::scan_fwd_kernel<blr::IoBF16, blr::MathFast><<<grid, block, 0, st>>>(a);
+  // Clear the forward header (tickets, counters, error word), empty the
+  // forward records, precompute k = -c softplus(Lambda).
+  BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fagg,
+                      plan.off_bagg - plan.off_fagg, reinterpret_cast<float*>(w + plan.off_k),
+                      lambda, desc->D, desc->c, st));
+  blr::FwdArgs a{plan, x, gate_logits, h0, h, h_last, w};
+  const int threads = plan.nwarps * 32;
+  unsigned grid = 1;
+  if (desc->io == BLR_F32) {
+    auto k = blr::scan_fwd_kernel<float, 4, blr::MathPrecise>;
+    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_f, &grid));
+    k<<<grid, threads, 0, st>>>(a);
+  } else {
+    auto k = blr::scan_fwd_kernel<__nv_bfloat16, 4, blr::MathFast>;
+    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_f, &grid));
+    k<<<grid, threads, 0, st>>>(a);
+  }
   return cuda_check(cudaGetLastError(), "launch scan_fwd_kernel");
 }
 
@@ -161,15 +200,23 @@ blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_la
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
-  // Clear the backward header, the dLambda partial sums and the backward flags.
-  BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_bhdr, 0, plan.off_fagg - plan.off_bhdr, st),
-                     "clear backward workspace"));
+  // Clear the backward header and the dLambda partial sums, empty the backward
+  // records (the forward's records stay: they hold the carries).
+  BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, w + plan.off_bagg,
+                      plan.bytes - plan.off_bagg, reinterpret_cast<float*>(w + plan.off_k), lambda,
+                      desc->D, desc->c, st));
   blr::BwdArgs a{plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda, dh0, w};
-  const dim3 grid((unsigned)plan.n_tiles), block = scan_block(plan);
-  if (desc->io == BLR_F32)
-    blr::scan_bwd_kernel<blr::IoF32, blr::MathPrecise><<<grid, block, 0, st>>>(a);
-  else
-    blr::scan_bwd_kernel<blr::IoBF16, blr::MathFast><<<grid, block, 0, st>>>(a);
+  const int threads = plan.nwarps * 32;
+  unsigned grid = 1;
+  if (desc->io == BLR_F32) {
+    auto k = blr::scan_bwd_kernel<float, 4, blr::MathPrecise>;
+    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_b, &grid));
+    k<<<grid, threads, 0, st>>>(a);
+  } else {
+    auto k = blr::scan_bwd_kernel<__nv_bfloat16, 4, blr::MathFast>;
+    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_b, &grid));
+    k<<<grid, threads, 0, st>>>(a);
+  }
   return cuda_check(cudaGetLastError(), "launch scan_bwd_kernel");
 }
 
@@ -188,7 +235,7 @@ blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_
   BLR_TRY(need(lambda, "lambda", 16));
   BLR_TRY(need(h_t, "h_t", 16));
   constexpr int kRows = 4;
-  const int vec = (io == BLR_F32) ? blr::IoF32::kVec : blr::IoBF16::kVec;
+  const int vec = (io == BLR_F32) ? 4 : 8;
   const int64_t nvec = D / vec;
   const int bx = (int)(nvec < 64 ? nvec : 64);
   const int by = 256 / bx;
@@ -196,13 +243,13 @@ blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_
   const int64_t rows_per_block = (int64_t)by * kRows;
   const int64_t n_rgroups = (B + rows_per_block - 1) / rows_per_block;
   if (n_vgroups * n_rgroups >= ((int64_t)1 << 31)) return fail(BLR_ERR_UNSUPPORTED, "grid too large");
-  blr::StepArgs a{B, D, c, kRows, n_vgroups, h_prev, x_t, gate_logits_t, lambda, h_t};
+  blr::StepArgs a{B, D, c, n_vgroups, h_prev, x_t, gate_logits_t, lambda, h_t};
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const dim3 grid((unsigned)(n_vgroups * n_rgroups)), block((unsigned)bx, (unsigned)by);
   if (io == BLR_F32)
-    blr::step_kernel<blr::IoF32, blr::MathPrecise, kRows><<<grid, block, 0, st>>>(a);
+    blr::step_kernel<float, 4, blr::MathPrecise, kRows><<<grid, block, 0, st>>>(a);
   else
-    blr::step_kernel<blr::IoBF16, blr::MathFast, kRows><<<grid, block, 0, st>>>(a);
+    blr::step_kernel<__nv_bfloat16, 8, blr::MathFast, kRows><<<grid, block, 0, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch step_kernel");
 }
 

@@ -1,30 +1,37 @@
 // BD-LRU scan kernels for sm_103a: forward scan, backward reverse scan,
-// single recurrent step. All are memory-bound elementwise scans: no tensor
-// cores, 16-byte loads and stores along the channels, gate arithmetic fused
-// into the load, float32 state.
+// single recurrent step, and the per-call preparation kernel. The path is
+// elementwise and memory-bound: no tensor cores; 16-byte (or 8-byte) accesses
+// along the channels, the gate arithmetic fused into the loads, float32 state.
 //
-// Scan structure (one thread block per tile of ttile steps x dblk channels):
-//   1. each thread loads its tc x vec elements, computes the gates and folds
-//      its chunk into one affine map h -> A h + U (serial, in registers);
-//   2. warp 0 turns the chunk maps of every channel into exclusive prefix maps
-//      (shared memory) and the tile's total map;
-//   3. warp 0 chains the tile to its predecessors in time with a decoupled
-//      look-back over per-tile records in the workspace (bounded waits);
-//   4. every thread applies its prefix map to the tile's carry and re-runs its
+// Scan structure. Persistent thread blocks take tiles (tsteps time steps x CH
+// channels of one batch row) from an atomic ticket counter, time-major, so a
+// tile only ever waits for tiles handed out before it. For one tile:
+//   1. every lane loads its kTc steps x VEC channels, computes the gates and
+//      folds its chunk into one affine map h -> A h + U, serially in registers;
+//   2. the kNtl lanes of a warp that share channels combine their maps with
+//      warp shuffles into exclusive prefix maps and a warp map;
+//   3. warp 0 combines the warp maps (shared memory) into the tile map and
+//      chains the tile to the tiles before it with a decoupled look-back: one
+//      lane per predecessor reads its status flag, a ballot finds the nearest
+//      published prefix, and the aggregates in between are folded in;
+//   4. every lane applies its prefix maps to the tile's carry and re-runs its
 //      chunk from the true state, writing the outputs.
-// Tiles are handed out in launch order by an atomic ticket, time-major, so a
-// block only ever waits for blocks that started before it.
+// Shared state is double-buffered by tile parity, so one barrier before and
+// one after warp 0's part are the only block-wide synchronisation per tile.
 #pragma once
+
+#include <limits.h>
 
 #include "blr_device.cuh"
 
 namespace blr {
 
+constexpr unsigned kFull = 0xffffffffu;
+
 struct FwdArgs {
   Plan p;
   const void* x;
   const void* gl;
-  const float* lambda;
   const float* h0;
   void* h;
   float* h_last;
@@ -49,8 +56,7 @@ struct BwdArgs {
 struct StepArgs {
   int64_t B, D;
   float c;
-  int rows;          // batch rows per thread
-  int64_t n_vgroups; // blocks along the channel vectors
+  int64_t n_vgroups;  // blocks along the channel vectors
   const float* h_prev;
   const void* x;
   const void* gl;
@@ -58,197 +64,347 @@ struct StepArgs {
   float* h_t;
 };
 
-constexpr int kCpl = kMaxDblk / 32;  // channels per lane of warp 0
+// ------------------------------------------------------------ preparation
+//
+// Clears the counters of a scan (tickets, exits, partial sums), fills its
+// look-back records with the empty pattern, and writes k[d] = -c softplus(Lambda_d).
+
+__global__ void prep_kernel(uint32_t* zero, int64_t zero_words, uint4* fill, int64_t fill_vec4,
+                            float* k, const float* lambda, int64_t D, float c) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (int64_t i = i0; i < zero_words; i += stride) zero[i] = 0u;
+  const uint4 empty = make_uint4(kEmpty, kEmpty, kEmpty, kEmpty);
+  for (int64_t i = i0; i < fill_vec4; i += stride) fill[i] = empty;
+  for (int64_t d = i0; d < D; d += stride) k[d] = decay_rate(c, lambda[d]);
+}
+
+// ------------------------------------------------------- warp-level scans
+//
+// Lane layout: lane = tcl * kNvl + cv. The kNtl lanes with the same cv hold
+// consecutive chunks in time of the same channels.
+
+// Turns each lane's chunk map (A, U) into the exclusive prefix map of the
+// chunks before it in the warp (ea, eu), and returns the warp's map (ta, tu).
+template <int V>
+__device__ __forceinline__ void warp_prefix(float (&A)[V], float (&U)[V], int tcl, int cv,
+                                            float (&ea)[V], float (&eu)[V], float (&ta)[V],
+                                            float (&tu)[V]) {
+#pragma unroll
+  for (int off = 1; off < kNtl; off <<= 1) {
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const float pa = __shfl_up_sync(kFull, A[v], off * kNvl);
+      const float pu = __shfl_up_sync(kFull, U[v], off * kNvl);
+      if (tcl >= off) {  // (this . earlier) = (A pa, A pu + U)
+        U[v] = fmaf(A[v], pu, U[v]);
+        A[v] *= pa;
+      }
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    ea[v] = __shfl_up_sync(kFull, A[v], kNvl);
+    eu[v] = __shfl_up_sync(kFull, U[v], kNvl);
+    if (tcl == 0) {
+      ea[v] = 1.0f;
+      eu[v] = 0.0f;
+    }
+    ta[v] = __shfl_sync(kFull, A[v], (kNtl - 1) * kNvl + cv);
+    tu[v] = __shfl_sync(kFull, U[v], (kNtl - 1) * kNvl + cv);
+  }
+}
+
+// The same from the end of the warp's time range: (sa, sw) maps the value
+// entering after the warp's last step to the value entering after this
+// lane's chunk; (ta, tw) is the warp's map.
+template <int V>
+__device__ __forceinline__ void warp_suffix(float (&A)[V], float (&W)[V], int tcl, int cv,
+                                            float (&sa)[V], float (&sw)[V], float (&ta)[V],
+                                            float (&tw)[V]) {
+#pragma unroll
+  for (int off = 1; off < kNtl; off <<= 1) {
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const float na = __shfl_down_sync(kFull, A[v], off * kNvl);
+      const float nw = __shfl_down_sync(kFull, W[v], off * kNvl);
+      if (tcl + off < kNtl) {  // (this . later) = (A na, A nw + W)
+        W[v] = fmaf(A[v], nw, W[v]);
+        A[v] *= na;
+      }
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    sa[v] = __shfl_down_sync(kFull, A[v], kNvl);
+    sw[v] = __shfl_down_sync(kFull, W[v], kNvl);
+    if (tcl == kNtl - 1) {
+      sa[v] = 1.0f;
+      sw[v] = 0.0f;
+    }
+    ta[v] = __shfl_sync(kFull, A[v], cv);
+    tw[v] = __shfl_sync(kFull, W[v], cv);
+  }
+}
+
+// ---------------------------------------------------------------- look-back
+//
+// Run by each lane of warp 0 for its own channel. Predecessor i (i = 0 is the
+// adjacent tile in scan order) has its records at agg[i * step] and
+// pre[i * step]. A window of kLookWindow predecessors is read in one round
+// trip; the walk folds aggregates (nearest first) until it meets a published
+// prefix. The farthest predecessor (i = nprev - 1, the first tile of the
+// chain) publishes only a prefix, so the walk always ends.
+__device__ __forceinline__ float lookback(const unsigned long long* agg, const uint32_t* pre,
+                                          int64_t step, int64_t nprev, uint32_t* err) {
+  float ea = 1.0f, eu = 0.0f;  // fold of the predecessors walked so far
+  int64_t i = 0;
+  for (;;) {
+    uint32_t pr[kLookWindow];
+    unsigned long long ag[kLookWindow];
+#pragma unroll
+    for (int q = 0; q < kLookWindow; ++q) {
+      pr[q] = kEmpty;
+      ag[q] = ~0ull;
+      if (i + q < nprev) {
+        pr[q] = ld_record(pre + (i + q) * step);
+        ag[q] = ld_record(agg + (i + q) * step);
+      }
+    }
+    int adv = kLookWindow;
+    bool open = true, wait = false;
+#pragma unroll
+    for (int q = 0; q < kLookWindow; ++q) {
+      if (open) {
+        if (pr[q] != kEmpty) return fmaf(ea, __uint_as_float(pr[q]), eu);
+        if (agg_empty(ag[q])) {  // published nothing yet: wait for it, then re-read from it
+          open = false;
+          wait = true;
+          adv = q;
+        } else {
+          eu = fmaf(ea, __uint_as_float((uint32_t)(ag[q] >> 32)), eu);
+          ea *= __uint_as_float((uint32_t)ag[q]);
+        }
+      }
+    }
+    if (wait && !wait_record(pre + (i + adv) * step, agg + (i + adv) * step, err, kWaitTimeoutNs))
+      return eu;  // the wait expired (recorded): finish with what is known
+    i += adv;
+  }
+}
+
+// ------------------------------------------------------------ tile tickets
+//
+// A ticket is decoded once, by the lane that draws it, into the tile's
+// position; blocks keep the decoded tiles in a three-slot ring: the tile being
+// finished, the next one (whose inputs are already being loaded) and the one
+// after (drawn during the current tile).
+
+struct TileCoord {
+  int64_t tile;   // the ticket; >= the tile count means no tile
+  int64_t tt;     // time tile
+  int64_t cidx;   // channel group in [0, B * groups per row)
+  int64_t b;      // batch row
+  int64_t dbase;  // first channel of the group
+};
+
+__device__ __forceinline__ TileCoord decode_tile(int64_t tile, int64_t n_tiles, int64_t n_c,
+                                                 int64_t n_cg, int ch, int64_t n_t, bool reverse) {
+  TileCoord c;
+  c.tile = tile;
+  c.tt = c.cidx = c.b = c.dbase = 0;
+  if (tile < n_tiles) {
+    const int64_t q = tile / n_c;
+    c.tt = reverse ? n_t - 1 - q : q;  // the backward hands tiles out from the end
+    c.cidx = tile - q * n_c;
+    c.b = c.cidx / n_cg;
+    c.dbase = (c.cidx - c.b * n_cg) * ch;
+  }
+  return c;
+}
 
 // ---------------------------------------------------------------- forward scan
 
-template <class IO, class M>
-__global__ void __launch_bounds__(256) scan_fwd_kernel(const FwdArgs a) {
-  constexpr int VEC = IO::kVec;
-  constexpr int TC = kTc;
-  using T = typename IO::T;
+template <typename T, int VEC, class M>
+__global__ void __launch_bounds__(kMaxWarps * 32, 3) scan_fwd_kernel(const FwdArgs a) {
+  using IO = Io<T, VEC>;
+  using Raw = typename IO::Raw;
+  constexpr int CH = kNvl * VEC;
+  static_assert(CH == 32, "warp 0 handles one channel per lane");
   const Plan& p = a.p;
 
-  __shared__ float2 s_map[kMaxNt][kMaxDblk];  // chunk map, then exclusive prefix map
-  __shared__ float s_carry[kMaxDblk];
-  __shared__ uint32_t s_ticket;
+  __shared__ float2 s_wmap[2][kMaxWarps][CH];  // warp maps, then warp prefix maps
+  __shared__ float s_carry[2][CH];
+  __shared__ TileCoord s_tc[3];
 
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
-  uint32_t* flags = reinterpret_cast<uint32_t*>(a.ws + p.off_fflags);
-  float2* agg = reinterpret_cast<float2*>(a.ws + p.off_fagg);
-  float* pre = reinterpret_cast<float*>(a.ws + p.off_fpre);
-
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  const int tid = ty * p.nv + tx;
-  if (tid == 0) s_ticket = atomicAdd(&fh->ticket, 1u);
-  __syncthreads();
-  const int64_t rec = s_ticket;
-  const int64_t it = rec / p.n_c;
-  const int64_t cb = rec - it * p.n_c;
-  const int64_t b = cb / p.n_dblk;
-  const int64_t dbase = (cb - b * p.n_dblk) * p.dblk;
-  const int cl = tx * VEC;
-  const int64_t d0 = dbase + cl;
-  const bool ch_ok = d0 < p.D;
-  const int64_t t0 = it * p.ttile + (int64_t)ty * TC;
-  if (rec == 0 && tid == 0) fh->tag = p.tag;
-
+  unsigned long long* agg = reinterpret_cast<unsigned long long*>(a.ws + p.off_fagg);
+  uint32_t* pre = reinterpret_cast<uint32_t*>(a.ws + p.off_fpre);
+  const float* kd = reinterpret_cast<const float*>(a.ws + p.off_k);
   const T* x = static_cast<const T*>(a.x);
   const T* gl = static_cast<const T*>(a.gl);
+  T* h = static_cast<T*>(a.h);
 
-  float k[VEC];
-#pragma unroll
-  for (int j = 0; j < VEC; j += 4) {
-    float lam[4] = {0.f, 0.f, 0.f, 0.f};
-    if (ch_ok) load_f32x4(a.lambda + d0 + j, lam);
-#pragma unroll
-    for (int v = 0; v < 4; ++v) k[j + v] = decay_rate(p.c, lam[v]);
-  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cv = lane % kNvl, tcl = lane / kNvl;
+  const int64_t BD = p.B * p.D;
+  const int64_t lane_t = (int64_t)warp * kWarpSteps + tcl * kTc;  // first step within a tile
 
-  // 1. loads (all issued before any use), gates, chunk map.
-  float xv[TC][VEC], rv[TC][VEC], iv[TC][VEC];
-#pragma unroll
-  for (int s = 0; s < TC; ++s) {
-    const int64_t t = t0 + s;
-    if (ch_ok && t < p.L) {
-      const int64_t row = b * p.L + t;
-      IO::load(x + row * p.D + d0, xv[s]);
-      IO::load(gl + row * 2 * p.D + d0, rv[s]);
-      IO::load(gl + row * 2 * p.D + p.D + d0, iv[s]);
-    }
-  }
-  float al[TC][VEC], u[TC][VEC];
-#pragma unroll
-  for (int s = 0; s < TC; ++s) {
-    const bool ok = ch_ok && (t0 + s < p.L);
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      if (ok) {
-        float r, i, alpha, q;
-        gates<M>(k[v], rv[s][v], iv[s][v], r, i, alpha, q);
-        al[s][v] = alpha;
-        u[s][v] = M::sqrt(q) * i * xv[s][v];
-      } else {  // outside the sequence or the channels: the identity map
-        al[s][v] = 1.0f;
-        u[s][v] = 0.0f;
-      }
-    }
-  }
-#pragma unroll
-  for (int v = 0; v < VEC; ++v) {
-    float A = 1.0f, U = 0.0f;
-#pragma unroll
-    for (int s = 0; s < TC; ++s) {
-      U = fmaf(al[s][v], U, u[s][v]);
-      A *= al[s][v];
-    }
-    s_map[ty][cl + v] = make_float2(A, U);
+  auto decode = [&](uint32_t t) {
+    return decode_tile((int64_t)t, p.n_tiles_f, p.n_c_f, p.n_cg_f, CH, p.n_t, false);
+  };
+  const bool drawer = threadIdx.x == blockDim.x - 1;  // draws the tickets
+  if (drawer) {
+    s_tc[0] = decode(atomicAdd(&fh->ticket, 1u));
+    s_tc[1] = decode(atomicAdd(&fh->ticket, 1u));
   }
   __syncthreads();
 
-  // 2.-3. warp 0: prefix maps, tile map, look-back, tile prefix.
-  if (tid < 32) {
-    uint32_t* err = &fh->err;
-    float tA[kCpl], tU[kCpl], carry[kCpl];
+  // The raw inputs of the next tile, in flight while the current one finishes.
+  Raw nx[kTc], nr[kTc], ni[kTc];
+  float nk[VEC];
+  auto fetch = [&](const TileCoord& c) {
+    const int64_t d0 = c.dbase + cv * VEC;
+    const int64_t t0 = c.tt * p.tsteps + lane_t;
 #pragma unroll
-    for (int j = 0; j < kCpl; ++j) {
-      const int ch = tid + 32 * j;
-      float pa = 1.0f, pu = 0.0f;
-      if (ch < p.dblk) {
-        for (int m = 0; m < p.nt; ++m) {
-          const float2 e = s_map[m][ch];
-          s_map[m][ch] = make_float2(pa, pu);
-          pu = fmaf(e.x, pu, e.y);
-          pa *= e.x;
+    for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+    if (d0 < p.D) {
+      load_f32<VEC>(kd + d0, nk);
+      const T* px = x + (c.b * p.L + t0) * p.D + d0;
+      const T* pg = gl + (c.b * p.L + t0) * 2 * p.D + d0;
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        if (t0 + s < p.L) {
+          nx[s] = IO::load_raw(px + s * p.D);
+          nr[s] = IO::load_raw(pg + s * 2 * p.D);
+          ni[s] = IO::load_raw(pg + s * 2 * p.D + p.D);
         }
       }
-      tA[j] = pa;
-      tU[j] = pu;
-      carry[j] = 0.0f;
     }
-    if (it == 0) {
-#pragma unroll
-      for (int j = 0; j < kCpl; ++j) {
-        const int ch = tid + 32 * j;
-        if (ch < p.dblk && dbase + ch < p.D && a.h0 != nullptr) carry[j] = a.h0[b * p.D + dbase + ch];
-      }
-    } else {
-#pragma unroll
-      for (int j = 0; j < kCpl; ++j) {
-        const int ch = tid + 32 * j;
-        if (ch < p.dblk) __stcg(&agg[rec * p.dblk + ch], make_float2(tA[j], tU[j]));
-      }
-      __threadfence();
-      __syncwarp();
-      if (tid == 0) st_release(&flags[rec], kFlagAggregate);
-      float ea[kCpl], eu[kCpl];
-#pragma unroll
-      for (int j = 0; j < kCpl; ++j) { ea[j] = 1.0f; eu[j] = 0.0f; }
-      int64_t q = rec - p.n_c;  // the same channel block, one tile earlier
-      for (;;) {
-        const uint32_t f = wait_flag(&flags[q], err, kWaitTimeoutNs);
-        if (f != kFlagAggregate) {  // a prefix (or 0: the wait expired, carry 0)
-#pragma unroll
-          for (int j = 0; j < kCpl; ++j) {
-            const int ch = tid + 32 * j;
-            if (ch < p.dblk) {
-              const float pv = (f == kFlagPrefix) ? __ldcg(&pre[q * p.dblk + ch]) : 0.0f;
-              carry[j] = fmaf(ea[j], pv, eu[j]);
-            }
-          }
-          break;
-        }
-#pragma unroll
-        for (int j = 0; j < kCpl; ++j) {
-          const int ch = tid + 32 * j;
-          if (ch < p.dblk) {
-            const float2 g = __ldcg(&agg[q * p.dblk + ch]);
-            eu[j] = fmaf(ea[j], g.y, eu[j]);
-            ea[j] *= g.x;
-          }
-        }
-        q -= p.n_c;
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < kCpl; ++j) {
-      const int ch = tid + 32 * j;
-      if (ch < p.dblk) {
-        const float incl = fmaf(tA[j], carry[j], tU[j]);
-        __stcg(&pre[rec * p.dblk + ch], incl);
-        s_carry[ch] = carry[j];
-        if (it == p.n_t - 1 && a.h_last != nullptr && dbase + ch < p.D)
-          a.h_last[b * p.D + dbase + ch] = incl;
-      }
-    }
-    __threadfence();
-    __syncwarp();
-    if (tid == 0) st_release(&flags[rec], kFlagPrefix);
-  }
-  __syncthreads();
+  };
+  if (s_tc[0].tile < p.n_tiles_f) fetch(s_tc[0]);
 
-  // 4. re-run the chunk from its true starting state.
-  if (a.h != nullptr && ch_ok) {
-    T* h = static_cast<T*>(a.h);
-    float hs[VEC];
+  for (int it = 0;; ++it) {
+    const int buf = it & 1;
+    const TileCoord tc = s_tc[it % 3];
+    if (tc.tile >= p.n_tiles_f) break;
+    const int64_t d0 = tc.dbase + cv * VEC;
+    const bool ch_ok = d0 < p.D;
+    const int64_t t0 = tc.tt * p.tsteps + lane_t;
+    // the ticket after next: drawn now, decoded before the barrier
+    const uint32_t ticket = drawer ? atomicAdd(&fh->ticket, 1u) : 0u;
+
+    // 1. gates and chunk map from the raw registers
+    float k[VEC];
 #pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      const float2 m = s_map[ty][cl + v];
-      hs[v] = fmaf(m.x, s_carry[cl + v], m.y);
-    }
+    for (int v = 0; v < VEC; ++v) k[v] = nk[v];
+    float al[kTc][VEC], u[kTc][VEC];
 #pragma unroll
-    for (int s = 0; s < TC; ++s) {
-      float out[VEC];
+    for (int s = 0; s < kTc; ++s) {
+      const bool ok = ch_ok && t0 + s < p.L;
+      float xv[VEC], rv[VEC], iv[VEC];
+      IO::unpack(nx[s], xv);
+      IO::unpack(nr[s], rv);
+      IO::unpack(ni[s], iv);
 #pragma unroll
       for (int v = 0; v < VEC; ++v) {
-        hs[v] = fmaf(al[s][v], hs[v], u[s][v]);
-        out[v] = hs[v];
+        if (ok) {
+          const float r = M::sigmoid(rv[v]);
+          const float i = M::sigmoid(iv[v]);
+          const float e = M::expm1_nonpos(k[v] * r);
+          al[s][v] = 1.0f + e;
+          u[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[v];
+        } else {  // outside the sequence or the channels: the identity map
+          al[s][v] = 1.0f;
+          u[s][v] = 0.0f;
+        }
       }
-      const int64_t t = t0 + s;
-      if (t < p.L) IO::store(h + (b * p.L + t) * p.D + d0, out);
+    }
+    // the next tile's inputs start moving now
+    {
+      const TileCoord nc = s_tc[(it + 1) % 3];
+      if (nc.tile < p.n_tiles_f) fetch(nc);
+    }
+    float A[VEC], U[VEC];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+      A[v] = 1.0f;
+      U[v] = 0.0f;
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        U[v] = fmaf(al[s][v], U[v], u[s][v]);
+        A[v] *= al[s][v];
+      }
+    }
+    // 2. warp prefix maps
+    float ea[VEC], eu[VEC], wa[VEC], wu[VEC];
+    warp_prefix<VEC>(A, U, tcl, cv, ea, eu, wa, wu);
+    if (tcl == kNtl - 1) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) s_wmap[buf][warp][cv * VEC + v] = make_float2(wa[v], wu[v]);
+    }
+    if (drawer) s_tc[(it + 2) % 3] = decode(ticket);
+    __syncthreads();
+
+    // 3. warp 0, one lane per channel: tile map, look-back, tile prefix
+    if (warp == 0) {
+      const int ch = lane;
+      const bool cval = tc.dbase + ch < p.D;
+      float pa = 1.0f, pu = 0.0f;
+      for (int w = 0; w < p.nwarps; ++w) {
+        const float2 e = s_wmap[buf][w][ch];
+        s_wmap[buf][w][ch] = make_float2(pa, pu);
+        pu = fmaf(e.x, pu, e.y);
+        pa *= e.x;
+      }
+      float carry = 0.0f;
+      if (cval) {
+        const int64_t rec = tc.tt * BD + tc.b * p.D + tc.dbase + ch;
+        if (tc.tt == 0) {
+          if (a.h0 != nullptr) carry = a.h0[tc.b * p.D + tc.dbase + ch];
+        } else {
+          st_record(&agg[rec], pack_agg(pa, pu));
+          carry = lookback(agg + rec - BD, pre + rec - BD, -BD, tc.tt, &fh->err);
+        }
+        const float incl = fmaf(pa, carry, pu);
+        st_record(&pre[rec], __float_as_uint(incl));
+        if (tc.tt == p.n_t - 1 && a.h_last != nullptr) a.h_last[tc.b * p.D + tc.dbase + ch] = incl;
+      }
+      s_carry[buf][ch] = carry;
+    }
+    __syncthreads();
+
+    // 4. re-run the chunk from its true starting state
+    if (h != nullptr && ch_ok) {
+      float hs[VEC];
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        const float2 wm = s_wmap[buf][warp][cv * VEC + v];
+        hs[v] = fmaf(ea[v], fmaf(wm.x, s_carry[buf][cv * VEC + v], wm.y), eu[v]);
+      }
+      T* ph = h + (tc.b * p.L + t0) * p.D + d0;
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        float out[VEC];
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) {
+          hs[v] = fmaf(al[s][v], hs[v], u[s][v]);
+          out[v] = hs[v];
+        }
+        if (t0 + s < p.L) IO::store(ph + s * p.D, out);
+      }
     }
   }
-  if (tid == 0) atomicAdd(&fh->done, 1u);
+  // The last block out marks the forward complete (for the backward's check).
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(&fh->exited, 1u) == gridDim.x - 1) {
+      fh->tag = p.tag;
+      __threadfence();
+      fh->complete = 1u;
+    }
+  }
 }
 
 // ------------------------------------------------------- backward reverse scan
@@ -264,283 +420,270 @@ __global__ void __launch_bounds__(256) scan_fwd_kernel(const FwdArgs a) {
 //   dLambda += dl (-c r) sigmoid(Lambda)      (summed over b, t)
 // h_{t-1} is rebuilt from the forward's per-tile carries, not read from h.
 
-template <class IO, class M>
-__global__ void __launch_bounds__(256) scan_bwd_kernel(const BwdArgs a) {
-  constexpr int VEC = IO::kVec;
-  constexpr int TC = kTc;
-  using T = typename IO::T;
+template <typename T, int VEC, class M>
+__global__ void __launch_bounds__(kMaxWarps * 32, sizeof(T) == 4 ? 2 : 3)
+    scan_bwd_kernel(const BwdArgs a) {
+  using IO = Io<T, VEC>;
+  using Raw = typename IO::Raw;
+  constexpr int CH = kNvl * VEC;
+  static_assert(CH == 32, "warp 0 handles one channel per lane");
   const Plan& p = a.p;
 
-  __shared__ float s_a[kMaxNt][kMaxDblk];   // chunk prod alpha -> prefix map A
-  __shared__ float s_u[kMaxNt][kMaxDblk];   // chunk U          -> prefix map U
-  __shared__ float s_w[kMaxNt][kMaxDblk];   // chunk W          -> suffix map W
-  __shared__ float s_sa[kMaxNt][kMaxDblk];  //                  -> suffix map A
-  __shared__ float s_hc[kMaxDblk], s_wc[kMaxDblk];
-  __shared__ uint32_t s_ticket;
+  __shared__ float s_wa[2][kMaxWarps][CH];   // warp prod alpha -> warp prefix map A
+  __shared__ float s_wu[2][kMaxWarps][CH];   // warp U          -> warp prefix map U
+  __shared__ float s_ww[2][kMaxWarps][CH];   // warp W          -> warp suffix map W
+  __shared__ float s_ws[2][kMaxWarps][CH];   //                 -> warp suffix map A
+  __shared__ float s_hc[2][CH], s_wc[2][CH];
+  __shared__ TileCoord s_tc[3];
   __shared__ int s_flag;
 
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
   BwdHeader* bh = reinterpret_cast<BwdHeader*>(a.ws + p.off_bhdr);
-  uint32_t* flags = reinterpret_cast<uint32_t*>(a.ws + p.off_bflags);
-  float2* agg = reinterpret_cast<float2*>(a.ws + p.off_bagg);
-  float* pre = reinterpret_cast<float*>(a.ws + p.off_bpre);
+  unsigned long long* agg = reinterpret_cast<unsigned long long*>(a.ws + p.off_bagg);
+  uint32_t* pre = reinterpret_cast<uint32_t*>(a.ws + p.off_bpre);
   const float* fpre = reinterpret_cast<const float*>(a.ws + p.off_fpre);
+  const float* kd = reinterpret_cast<const float*>(a.ws + p.off_k);
   double* dlam_acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
-
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  const int tid = ty * p.nv + tx;
-  const int nthreads = p.nv * p.nt;
-  if (tid == 0) {
-    s_ticket = atomicAdd(&bh->ticket, 1u);
-    const bool ok = __ldcg(&fh->tag) == p.tag && __ldcg(&fh->done) == (uint32_t)p.n_tiles;
-    if (!ok) atomicOr(&fh->err, kErrWorkspace);
-    s_flag = ok;
-  }
-  __syncthreads();
-  if (!s_flag) return;  // no forward carries for this problem: write nothing
-  const int64_t ticket = s_ticket;
-  const int64_t it = p.n_t - 1 - ticket / p.n_c;  // tiles handed out from the end
-  const int64_t cb = ticket % p.n_c;
-  const int64_t rec = it * p.n_c + cb;
-  const int64_t b = cb / p.n_dblk;
-  const int64_t dbase = (cb - b * p.n_dblk) * p.dblk;
-  const int cl = tx * VEC;
-  const int64_t d0 = dbase + cl;
-  const bool ch_ok = d0 < p.D;
-  const int64_t t0 = it * p.ttile + (int64_t)ty * TC;
-
   const T* x = static_cast<const T*>(a.x);
   const T* gl = static_cast<const T*>(a.gl);
   const T* dh = static_cast<const T*>(a.dh);
-
-  float k[VEC];
-#pragma unroll
-  for (int j = 0; j < VEC; j += 4) {
-    float lam[4] = {0.f, 0.f, 0.f, 0.f};
-    if (ch_ok) load_f32x4(a.lambda + d0 + j, lam);
-#pragma unroll
-    for (int v = 0; v < 4; ++v) k[j + v] = decay_rate(p.c, lam[v]);
-  }
-
-  // 1. loads, gates, chunk maps of both directions.
-  float xv[TC][VEC], rv[TC][VEC], iv[TC][VEC], gv[TC][VEC];
-#pragma unroll
-  for (int s = 0; s < TC; ++s) {
-    const int64_t t = t0 + s;
-    if (ch_ok && t < p.L) {
-      const int64_t row = b * p.L + t;
-      IO::load(dh + row * p.D + d0, gv[s]);
-      IO::load(x + row * p.D + d0, xv[s]);
-      IO::load(gl + row * 2 * p.D + d0, rv[s]);
-      IO::load(gl + row * 2 * p.D + p.D + d0, iv[s]);
-    }
-  }
-  // Per element kept for the last pass: alpha, u, beta = n i, c2 = alpha u / q,
-  // ui = u (1 - i), r, and dh (then g).
-  float al[TC][VEC], u[TC][VEC], bt[TC][VEC], c2[TC][VEC], ui[TC][VEC], rr[TC][VEC];
-#pragma unroll
-  for (int s = 0; s < TC; ++s) {
-    const bool ok = ch_ok && (t0 + s < p.L);
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      if (ok) {
-        float r, i, alpha, q;
-        gates<M>(k[v], rv[s][v], iv[s][v], r, i, alpha, q);
-        const float beta = M::sqrt(q) * i;
-        const float uu = beta * xv[s][v];
-        al[s][v] = alpha;
-        u[s][v] = uu;
-        bt[s][v] = beta;
-        c2[s][v] = M::div(alpha * uu, q);
-        ui[s][v] = uu * (1.0f - i);
-        rr[s][v] = r;
-      } else {
-        al[s][v] = 1.0f;
-        u[s][v] = 0.0f;
-        bt[s][v] = 0.0f;
-        c2[s][v] = 0.0f;
-        ui[s][v] = 0.0f;
-        rr[s][v] = 0.0f;
-        gv[s][v] = 0.0f;
-      }
-    }
-  }
-#pragma unroll
-  for (int v = 0; v < VEC; ++v) {
-    float A = 1.0f, U = 0.0f, W = 0.0f;
-#pragma unroll
-    for (int s = 0; s < TC; ++s) {
-      U = fmaf(al[s][v], U, u[s][v]);
-      A *= al[s][v];            // prod of alpha up to and including s
-      W = fmaf(A, gv[s][v], W); // w at the chunk start from a zero carry
-    }
-    s_a[ty][cl + v] = A;
-    s_u[ty][cl + v] = U;
-    s_w[ty][cl + v] = W;
-  }
-  __syncthreads();
-
-  // 2.-3. warp 0.
-  if (tid < 32) {
-    uint32_t* err = &fh->err;
-    float tA[kCpl], tW[kCpl], hc[kCpl], wc[kCpl];
-#pragma unroll
-    for (int j = 0; j < kCpl; ++j) {
-      const int ch = tid + 32 * j;
-      float sa = 1.0f, su = 0.0f;
-      if (ch < p.dblk) {
-        for (int m = p.nt - 1; m >= 0; --m) {  // suffix maps, from the tile's end
-          const float A = s_a[m][ch], W = s_w[m][ch];
-          s_sa[m][ch] = sa;
-          s_w[m][ch] = su;
-          su = fmaf(A, su, W);
-          sa *= A;
-        }
-        float pa = 1.0f, pu = 0.0f;
-        for (int m = 0; m < p.nt; ++m) {       // prefix maps, from the tile's start
-          const float A = s_a[m][ch], U = s_u[m][ch];
-          s_a[m][ch] = pa;
-          s_u[m][ch] = pu;
-          pu = fmaf(A, pu, U);
-          pa *= A;
-        }
-      }
-      tA[j] = sa;
-      tW[j] = su;
-      hc[j] = 0.0f;
-      wc[j] = 0.0f;
-      if (ch < p.dblk && dbase + ch < p.D) {
-        if (it > 0)
-          hc[j] = __ldcg(&fpre[(rec - p.n_c) * p.dblk + ch]);
-        else if (a.h0 != nullptr)
-          hc[j] = a.h0[b * p.D + dbase + ch];
-      }
-    }
-    if (it == p.n_t - 1) {
-#pragma unroll
-      for (int j = 0; j < kCpl; ++j) {
-        const int ch = tid + 32 * j;
-        if (ch < p.dblk && dbase + ch < p.D && a.dh_last != nullptr)
-          wc[j] = a.dh_last[b * p.D + dbase + ch];
-      }
-    } else {
-#pragma unroll
-      for (int j = 0; j < kCpl; ++j) {
-        const int ch = tid + 32 * j;
-        if (ch < p.dblk) __stcg(&agg[rec * p.dblk + ch], make_float2(tA[j], tW[j]));
-      }
-      __threadfence();
-      __syncwarp();
-      if (tid == 0) st_release(&flags[rec], kFlagAggregate);
-      float ea[kCpl], eu[kCpl];
-#pragma unroll
-      for (int j = 0; j < kCpl; ++j) { ea[j] = 1.0f; eu[j] = 0.0f; }
-      int64_t q = rec + p.n_c;  // the same channel block, one tile later
-      for (;;) {
-        const uint32_t f = wait_flag(&flags[q], err, kWaitTimeoutNs);
-        if (f != kFlagAggregate) {
-#pragma unroll
-          for (int j = 0; j < kCpl; ++j) {
-            const int ch = tid + 32 * j;
-            if (ch < p.dblk) {
-              const float pv = (f == kFlagPrefix) ? __ldcg(&pre[q * p.dblk + ch]) : 0.0f;
-              wc[j] = fmaf(ea[j], pv, eu[j]);
-            }
-          }
-          break;
-        }
-#pragma unroll
-        for (int j = 0; j < kCpl; ++j) {
-          const int ch = tid + 32 * j;
-          if (ch < p.dblk) {
-            const float2 g = __ldcg(&agg[q * p.dblk + ch]);
-            eu[j] = fmaf(ea[j], g.y, eu[j]);
-            ea[j] *= g.x;
-          }
-        }
-        q += p.n_c;
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < kCpl; ++j) {
-      const int ch = tid + 32 * j;
-      if (ch < p.dblk) {
-        const float incl = fmaf(tA[j], wc[j], tW[j]);  // w at the tile's first step
-        __stcg(&pre[rec * p.dblk + ch], incl);
-        s_hc[ch] = hc[j];
-        s_wc[ch] = wc[j];
-        if (it == 0 && a.dh0 != nullptr && dbase + ch < p.D) a.dh0[b * p.D + dbase + ch] = incl;
-      }
-    }
-    __threadfence();
-    __syncwarp();
-    if (tid == 0) st_release(&flags[rec], kFlagPrefix);
-  }
-  __syncthreads();
-
-  // 4. g backwards through the chunk, then the gradients forwards with h_{t-1}.
-  float hs[VEC], wn[VEC], dl_r[VEC];
-#pragma unroll
-  for (int v = 0; v < VEC; ++v) {
-    hs[v] = fmaf(s_a[ty][cl + v], s_hc[cl + v], s_u[ty][cl + v]);
-    wn[v] = fmaf(s_sa[ty][cl + v], s_wc[cl + v], s_w[ty][cl + v]);
-    dl_r[v] = 0.0f;
-  }
-#pragma unroll
-  for (int s = TC - 1; s >= 0; --s) {
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      const float g = gv[s][v] + wn[v];
-      gv[s][v] = g;
-      wn[v] = al[s][v] * g;
-    }
-  }
   T* dx = static_cast<T*>(a.dx);
   T* dgl = static_cast<T*>(a.dgl);
-#pragma unroll
-  for (int s = 0; s < TC; ++s) {
-    float ox[VEC], orho[VEC], oiota[VEC];
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      const float g = gv[s][v];
-      const float dl = g * al[s][v] * (hs[v] - c2[s][v]);
-      const float r = rr[s][v];
-      orho[v] = dl * k[v] * (r - r * r);
-      oiota[v] = g * ui[s][v];
-      ox[v] = g * bt[s][v];
-      dl_r[v] = fmaf(dl, r, dl_r[v]);
-      hs[v] = fmaf(al[s][v], hs[v], u[s][v]);
-    }
-    const int64_t t = t0 + s;
-    if (ch_ok && t < p.L) {
-      const int64_t row = b * p.L + t;
-      IO::store(dx + row * p.D + d0, ox);
-      IO::store(dgl + row * 2 * p.D + d0, orho);
-      IO::store(dgl + row * 2 * p.D + p.D + d0, oiota);
-    }
-  }
 
-  // 5. dLambda: block sum over time chunks, float64 stripes, last block finishes.
-  __syncthreads();  // s_a is reused
-#pragma unroll
-  for (int v = 0; v < VEC; ++v) s_a[ty][cl + v] = dl_r[v];
-  __syncthreads();
-  if (ty == 0 && ch_ok) {
-    const int stripe = (int)(b % kStripes);
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      float sum = 0.0f;
-      for (int m = 0; m < p.nt; ++m) sum += s_a[m][cl + v];
-      atomicAdd(&dlam_acc[stripe * p.D + d0 + v], (double)sum);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cv = lane % kNvl, tcl = lane / kNvl;
+  const int64_t BD = p.B * p.D;
+  const int64_t lane_t = (int64_t)warp * kWarpSteps + tcl * kTc;
+
+  auto decode = [&](uint32_t t) {
+    return decode_tile((int64_t)t, p.n_tiles_b, p.n_c_b, p.n_cg_b, CH, p.n_t, true);
+  };
+  const bool drawer = threadIdx.x == blockDim.x - 1;  // draws the tickets
+  if (drawer) {
+    const bool ok = __ldcg(&fh->tag) == p.tag && __ldcg(&fh->complete) == 1u;
+    if (!ok) atomicOr(&fh->err, kErrWorkspace);
+    s_flag = ok;
+    if (ok) {
+      s_tc[0] = decode(atomicAdd(&bh->ticket, 1u));
+      s_tc[1] = decode(atomicAdd(&bh->ticket, 1u));
     }
   }
-  __threadfence();
   __syncthreads();
-  if (tid == 0) s_flag = (atomicAdd(&bh->done, 1u) == (uint32_t)(p.n_tiles - 1));
+  if (!s_flag) return;  // no forward carries for this problem: write nothing
+
+  Raw ng[kTc], nx[kTc], nr[kTc], ni[kTc];
+  float nk[VEC];
+  auto fetch = [&](const TileCoord& c) {
+    const int64_t d0 = c.dbase + cv * VEC;
+    const int64_t t0 = c.tt * p.tsteps + lane_t;
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+    if (d0 < p.D) {
+      load_f32<VEC>(kd + d0, nk);
+      const int64_t row = c.b * p.L + t0;
+      const T* pd = dh + row * p.D + d0;
+      const T* px = x + row * p.D + d0;
+      const T* pg = gl + row * 2 * p.D + d0;
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        if (t0 + s < p.L) {
+          ng[s] = IO::load_raw(pd + s * p.D);
+          nx[s] = IO::load_raw(px + s * p.D);
+          nr[s] = IO::load_raw(pg + s * 2 * p.D);
+          ni[s] = IO::load_raw(pg + s * 2 * p.D + p.D);
+        }
+      }
+    }
+  };
+  if (s_tc[0].tile < p.n_tiles_b) fetch(s_tc[0]);
+
+  for (int it = 0;; ++it) {
+    const int buf = it & 1;
+    const TileCoord tc = s_tc[it % 3];
+    if (tc.tile >= p.n_tiles_b) break;
+    const int64_t d0 = tc.dbase + cv * VEC;
+    const bool ch_ok = d0 < p.D;
+    const int64_t t0 = tc.tt * p.tsteps + lane_t;
+    // the ticket after next: drawn now, decoded before the barrier
+    const uint32_t ticket = drawer ? atomicAdd(&bh->ticket, 1u) : 0u;
+
+    // 1. gates kept as E = expm1(l), r, i (with x and dh); chunk maps of both directions
+    float k[VEC];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) k[v] = nk[v];
+    float xv[kTc][VEC], rv[kTc][VEC], iv[kTc][VEC], gv[kTc][VEC], ev[kTc][VEC];
+    float A[VEC], U[VEC], W[VEC];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+      A[v] = 1.0f;
+      U[v] = 0.0f;
+      W[v] = 0.0f;
+    }
+#pragma unroll
+    for (int s = 0; s < kTc; ++s) {
+      const bool ok = ch_ok && t0 + s < p.L;
+      IO::unpack(ng[s], gv[s]);
+      IO::unpack(nx[s], xv[s]);
+      IO::unpack(nr[s], rv[s]);
+      IO::unpack(ni[s], iv[s]);
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        if (ok) {
+          const float r = M::sigmoid(rv[s][v]);
+          const float i = M::sigmoid(iv[s][v]);
+          const float e = M::expm1_nonpos(k[v] * r);
+          const float alpha = 1.0f + e;
+          const float uu = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
+          rv[s][v] = r;
+          iv[s][v] = i;
+          ev[s][v] = e;
+          U[v] = fmaf(alpha, U[v], uu);
+          A[v] *= alpha;                      // prod of alpha up to and including s
+          W[v] = fmaf(A[v], gv[s][v], W[v]);  // w at the chunk start from a zero carry
+        } else {  // the identity: alpha = 1, no input, no upstream gradient
+          rv[s][v] = 0.0f;
+          iv[s][v] = 0.0f;
+          ev[s][v] = 0.0f;
+          gv[s][v] = 0.0f;
+          xv[s][v] = 0.0f;
+        }
+      }
+    }
+    {
+      const TileCoord nc = s_tc[(it + 1) % 3];
+      if (nc.tile < p.n_tiles_b) fetch(nc);
+    }
+    // 2. warp maps: h forwards (prefix), w backwards (suffix)
+    float A2[VEC];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) A2[v] = A[v];
+    float ea[VEC], eu[VEC], wa[VEC], wu[VEC], sa[VEC], sw[VEC], wa2[VEC], ww[VEC];
+    warp_prefix<VEC>(A, U, tcl, cv, ea, eu, wa, wu);
+    warp_suffix<VEC>(A2, W, tcl, cv, sa, sw, wa2, ww);
+    if (tcl == kNtl - 1) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        s_wa[buf][warp][cv * VEC + v] = wa[v];
+        s_wu[buf][warp][cv * VEC + v] = wu[v];
+      }
+    }
+    if (tcl == 0) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) s_ww[buf][warp][cv * VEC + v] = ww[v];
+    }
+    if (drawer) s_tc[(it + 2) % 3] = decode(ticket);
+    __syncthreads();
+
+    // 3. warp 0, one lane per channel: warp prefix / suffix maps, the h carry
+    //    from the forward, the w carry by look-back from the later tiles
+    if (warp == 0) {
+      const int ch = lane;
+      const bool cval = tc.dbase + ch < p.D;
+      float qa = 1.0f, qw = 0.0f;
+      for (int w = p.nwarps - 1; w >= 0; --w) {  // suffix maps first: they read s_wa
+        const float wA = s_wa[buf][w][ch], wW = s_ww[buf][w][ch];
+        s_ws[buf][w][ch] = qa;
+        s_ww[buf][w][ch] = qw;
+        qw = fmaf(wA, qw, wW);
+        qa *= wA;
+      }
+      float pa = 1.0f, pu = 0.0f;
+      for (int w = 0; w < p.nwarps; ++w) {
+        const float wA = s_wa[buf][w][ch], wU = s_wu[buf][w][ch];
+        s_wa[buf][w][ch] = pa;
+        s_wu[buf][w][ch] = pu;
+        pu = fmaf(wA, pu, wU);
+        pa *= wA;
+      }
+      float hc = 0.0f, wc = 0.0f;
+      if (cval) {
+        const int64_t rec = tc.tt * BD + tc.b * p.D + tc.dbase + ch;
+        if (tc.tt > 0)
+          hc = __ldcg(&fpre[rec - BD]);
+        else if (a.h0 != nullptr)
+          hc = a.h0[tc.b * p.D + tc.dbase + ch];
+        if (tc.tt == p.n_t - 1) {
+          if (a.dh_last != nullptr) wc = a.dh_last[tc.b * p.D + tc.dbase + ch];
+        } else {
+          st_record(&agg[rec], pack_agg(qa, qw));
+          wc = lookback(agg + rec + BD, pre + rec + BD, BD, p.n_t - 1 - tc.tt, &fh->err);
+        }
+        const float incl = fmaf(qa, wc, qw);  // w at the tile's first step
+        st_record(&pre[rec], __float_as_uint(incl));
+        if (tc.tt == 0 && a.dh0 != nullptr) a.dh0[tc.b * p.D + tc.dbase + ch] = incl;
+      }
+      s_hc[buf][ch] = hc;
+      s_wc[buf][ch] = wc;
+    }
+    __syncthreads();
+
+    // 4. g backwards through the chunk, then the gradients forwards with h_{t-1}
+    float hs[VEC], wn[VEC], dlr[VEC];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+      const int c = cv * VEC + v;
+      hs[v] = fmaf(ea[v], fmaf(s_wa[buf][warp][c], s_hc[buf][c], s_wu[buf][warp][c]), eu[v]);
+      wn[v] = fmaf(sa[v], fmaf(s_ws[buf][warp][c], s_wc[buf][c], s_ww[buf][warp][c]), sw[v]);
+      dlr[v] = 0.0f;
+    }
+#pragma unroll
+    for (int s = kTc - 1; s >= 0; --s) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        const float g = gv[s][v] + wn[v];
+        gv[s][v] = g;
+        wn[v] = (1.0f + ev[s][v]) * g;
+      }
+    }
+    const int64_t row0 = tc.b * p.L + t0;
+    T* pdx = dx + row0 * p.D + d0;
+    T* pdg = dgl + row0 * 2 * p.D + d0;
+#pragma unroll
+    for (int s = 0; s < kTc; ++s) {
+      float ox[VEC], orho[VEC], oiota[VEC];
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        const float e = ev[s][v], r = rv[s][v], i = iv[s][v], g = gv[s][v];
+        const float alpha = 1.0f + e;
+        const float q = -e * (2.0f + e);
+        const float beta = M::sqrt(q) * i;
+        const float uu = beta * xv[s][v];
+        const float c2 = (q > 0.0f) ? M::div(alpha * uu, q) : 0.0f;  // alpha i x / n
+        const float dl = g * alpha * (hs[v] - c2);
+        orho[v] = dl * k[v] * (r - r * r);
+        oiota[v] = g * uu * (1.0f - i);
+        ox[v] = g * beta;
+        dlr[v] = fmaf(dl, r, dlr[v]);
+        hs[v] = fmaf(alpha, hs[v], uu);
+      }
+      if (ch_ok && t0 + s < p.L) {
+        IO::store(pdx + s * p.D, ox);
+        IO::store(pdg + s * 2 * p.D, orho);
+        IO::store(pdg + s * 2 * p.D + p.D, oiota);
+      }
+    }
+    // 5. dLambda: sum over the warp's time lanes, one float64 add per channel
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+#pragma unroll
+      for (int off = 1; off < kNtl; off <<= 1) dlr[v] += __shfl_down_sync(kFull, dlr[v], off * kNvl);
+    }
+    if (tcl == 0 && ch_ok) {
+      double* acc = dlam_acc + (tc.b % kStripes) * p.D + d0;
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) atomicAdd(acc + v, (double)dlr[v]);
+    }
+  }
+  // The last block out turns the partial sums into dLambda.
   __syncthreads();
-  if (s_flag) {
+  if (threadIdx.x == 0) {
     __threadfence();
-    for (int64_t d = tid; d < p.D; d += nthreads) {
+    s_flag = (atomicAdd(&bh->exited, 1u) == gridDim.x - 1) ? 2 : 1;
+  }
+  __syncthreads();
+  if (s_flag == 2) {
+    __threadfence();
+    for (int64_t d = threadIdx.x; d < p.D; d += blockDim.x) {
       double sum = 0.0;
       for (int st = 0; st < kStripes; ++st) sum += __ldcg(&dlam_acc[st * p.D + d]);
       const double lam = (double)a.lambda[d];
@@ -551,27 +694,25 @@ __global__ void __launch_bounds__(256) scan_bwd_kernel(const BwdArgs a) {
 }
 
 // ------------------------------------------------------------ recurrent step
+//
+// h_t = alpha h_prev + beta x for B rows of D channels. A block covers
+// blockDim.x channel vectors of blockDim.y * ROWS rows; k = -c softplus(Lambda)
+// is computed once per channel per block.
 
-template <class IO, class M, int ROWS>
+template <typename T, int VEC, class M, int ROWS>
 __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
-  constexpr int VEC = IO::kVec;
-  using T = typename IO::T;
-  const int64_t nvec = a.D / VEC;
+  using IO = Io<T, VEC>;
+  __shared__ float s_k[64 * 8];
   const int64_t vg = blockIdx.x % a.n_vgroups;
   const int64_t rg = blockIdx.x / a.n_vgroups;
-  const int64_t vi = vg * blockDim.x + threadIdx.x;
-  if (vi >= nvec) return;
-  const int64_t d0 = vi * VEC;
+  const int64_t dblock = vg * blockDim.x * VEC;
+  const int tid = threadIdx.y * blockDim.x + threadIdx.x;
+  for (int j = tid; j < (int)blockDim.x * VEC; j += blockDim.x * blockDim.y)
+    if (dblock + j < a.D) s_k[j] = decay_rate(a.c, a.lambda[dblock + j]);
+  __syncthreads();
+  const int64_t d0 = dblock + threadIdx.x * VEC;
+  if (d0 >= a.D) return;
   const int64_t r0 = (rg * blockDim.y + threadIdx.y) * ROWS;
-
-  float k[VEC];
-#pragma unroll
-  for (int j = 0; j < VEC; j += 4) {
-    float lam[4];
-    load_f32x4(a.lambda + d0 + j, lam);
-#pragma unroll
-    for (int v = 0; v < 4; ++v) k[j + v] = decay_rate(a.c, lam[v]);
-  }
   const T* x = static_cast<const T*>(a.x);
   const T* gl = static_cast<const T*>(a.gl);
   float hp[ROWS][VEC], xv[ROWS][VEC], rv[ROWS][VEC], iv[ROWS][VEC];
@@ -579,11 +720,10 @@ __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
   for (int r = 0; r < ROWS; ++r) {
     const int64_t bb = r0 + r;
     if (bb < a.B) {
-#pragma unroll
-      for (int j = 0; j < VEC; j += 4) load_f32x4(a.h_prev + bb * a.D + d0 + j, &hp[r][j]);
-      IO::load(x + bb * a.D + d0, xv[r]);
-      IO::load(gl + bb * 2 * a.D + d0, rv[r]);
-      IO::load(gl + bb * 2 * a.D + a.D + d0, iv[r]);
+      load_f32<VEC>(a.h_prev + bb * a.D + d0, hp[r]);
+      IO::unpack(IO::load_raw(x + bb * a.D + d0), xv[r]);
+      IO::unpack(IO::load_raw(gl + bb * 2 * a.D + d0), rv[r]);
+      IO::unpack(IO::load_raw(gl + bb * 2 * a.D + a.D + d0), iv[r]);
     }
   }
 #pragma unroll
@@ -593,14 +733,16 @@ __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
       float out[VEC];
 #pragma unroll
       for (int v = 0; v < VEC; ++v) {
-        float rg_, i, alpha, q;
-        gates<M>(k[v], rv[r][v], iv[r][v], rg_, i, alpha, q);
-        out[v] = fmaf(alpha, hp[r][v], M::sqrt(q) * i * xv[r][v]);
+        const float k = s_k[threadIdx.x * VEC + v];
+        const float rr = M::sigmoid(rv[r][v]);
+        const float i = M::sigmoid(iv[r][v]);
+        const float e = M::expm1_nonpos(k * rr);
+        out[v] = fmaf(1.0f + e, hp[r][v], M::sqrt(-e * (2.0f + e)) * i * xv[r][v]);
       }
 #pragma unroll
       for (int j = 0; j < VEC; j += 4)
-        *reinterpret_cast<float4*>(a.h_t + bb * a.D + d0 + j) =
-            make_float4(out[j], out[j + 1], out[j + 2], out[j + 3]);
+        __stcs(reinterpret_cast<float4*>(a.h_t + bb * a.D + d0 + j),
+               make_float4(out[j], out[j + 1], out[j + 2], out[j + 3]));
     }
   }
 }
@@ -608,7 +750,7 @@ __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
 // ------------------------------------------------------------ bounded-wait test
 
 __global__ void selftest_wait_kernel(const uint32_t* flag, uint32_t* err, uint64_t timeout_ns) {
-  (void)wait_flag(flag, err, timeout_ns);
+  (void)wait_word(flag, err, timeout_ns);
 }
 
 }  // namespace blr

@@ -1,14 +1,16 @@
 // Tiling plan and workspace layout of the BD-LRU scan kernels (host and device).
 //
-// The (B, L, D) problem is cut into tiles of `ttile` time steps x `dblk`
-// channels of one batch row. One thread block scans one tile: thread (tx, ty)
-// owns channels [tx*vec, tx*vec + vec) of the block and the `tc` consecutive
-// time steps starting at ty*tc. Tiles of the same (batch row, channel block)
-// are chained along time with a single-pass decoupled look-back: each block
-// publishes its tile's aggregate (A = prod alpha, U = the tile's scan from a
-// zero state), then its inclusive prefix (the state at its last step) once the
-// carry from earlier tiles is known. The recurrence is the first-order linear
-// scan of Sec. 3.3, whose operator is (a2, u2) . (a1, u1) = (a2 a1, a2 u1 + u2).
+// The (B, L, D) problem is cut into tiles of `tsteps` consecutive time steps x
+// `CH` consecutive channels of one batch row. A thread block scans one tile at
+// a time (persistent blocks take tiles from an atomic ticket counter):
+//   lane (cv, tcl) of warp w owns channels [cv*VEC, cv*VEC + VEC) of the tile
+//   and the kTc steps starting at w*kWarpSteps + tcl*kTc.
+// Tiles of the same (batch row, channel group) are chained along time with a
+// single-pass decoupled look-back over per-tile, per-channel records: each
+// tile publishes its aggregate (A = prod alpha, U = its scan from a zero
+// state), then its inclusive prefix (the state after its last step). The recurrence is the
+// first-order linear scan of Sec. 3.3, whose operator on affine maps is
+// (a2, u2) . (a1, u1) = (a2 a1, a2 u1 + u2).
 #pragma once
 
 #include <stddef.h>
@@ -16,55 +18,63 @@
 
 namespace blr {
 
-constexpr int kMaxDblk = 64;       // channels per thread block
-constexpr int kMaxNt = 32;         // time chunks (threads along time) per block
-constexpr int kTc = 4;             // time steps per thread chunk
-constexpr int kTargetTile = 64;    // preferred time steps per tile
-constexpr int kStripes = 8;        // dlambda float64 partial-sum stripes
-constexpr size_t kAlign = 256;     // alignment of every workspace region
+constexpr int kNvl = 8;                    // lanes along channels (8 x 4 channels per row)
+constexpr int kNtl = 4;                    // lanes along time within a warp
+constexpr int kTc = 4;                     // time steps per lane
+constexpr int kWarpSteps = kNtl * kTc;     // time steps per warp
+constexpr int kMaxWarps = 4;               // warps (time sub-tiles) per tile
+constexpr int kStripes = 8;                // dlambda float64 partial-sum stripes
+constexpr size_t kAlign = 256;             // alignment of every workspace region
 
 // Error bits recorded in FwdHeader::err.
 constexpr uint32_t kErrTimeout = 1u;
 constexpr uint32_t kErrWorkspace = 2u;
-// Tile status flags of the look-back.
-constexpr uint32_t kFlagAggregate = 1u;
-constexpr uint32_t kFlagPrefix = 2u;
+// Per-tile records validate themselves: they are filled with this all-ones
+// pattern (a negative NaN with a full payload, which float arithmetic never
+// produces) before a scan, and a record is published by one 32- or 64-bit store.
+constexpr uint32_t kEmpty = 0xffffffffu;
+constexpr int kLookWindow = 4;     // predecessors read per round trip of the look-back
 
 // Upper bound of every inter-block wait.
 constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
 constexpr uint32_t kMaxWaitIters = 1u << 23;
 
-struct FwdHeader {     // zeroed before every forward
-  uint32_t ticket;     // tile tickets handed out (launch order of tiles)
-  uint32_t done;       // forward tiles completed
-  uint32_t err;        // error bits (timeouts of forward and backward, workspace misuse)
-  uint32_t tag;        // hash of the problem the carries belong to
+struct FwdHeader {     // cleared before every forward (by its prep kernel)
+  uint32_t ticket;     // tiles handed out
+  uint32_t exited;     // blocks that left the tile loop
+  uint32_t err;        // error bits (forward and backward timeouts, workspace misuse)
+  uint32_t tag;        // hash of the problem, written when the forward completed
+  uint32_t complete;   // 1 once every forward tile is done
+  uint32_t pad[3];
 };
 
-struct BwdHeader {     // zeroed before every backward
+struct BwdHeader {     // cleared before every backward
   uint32_t ticket;
-  uint32_t done;
+  uint32_t exited;
   uint32_t selftest_flag;  // a flag nothing sets (blr_selftest_wait_timeout)
-  uint32_t pad;
+  uint32_t pad[5];
 };
+
+// Channels per lane: 4 (a 16-byte float32 or an 8-byte bfloat16 vector), so a
+// lane holds 16 elements and a tile covers 8 x 4 = 32 channels.
+inline int fwd_vec(int) { return 4; }
+inline int bwd_vec(int) { return 4; }
 
 struct Plan {
   int64_t B, L, D;
   int io;           // 0 = float32, 1 = bfloat16
   float c;
-  int vec;          // channels per thread (one 16-byte vector)
-  int tc;           // time steps per thread chunk
-  int dblk;         // channels per tile
-  int nv;           // threads along channels = dblk / vec
-  int nt;           // threads along time
-  int64_t ttile;    // time steps per tile = tc * nt
-  int64_t n_dblk;   // channel blocks per batch row
-  int64_t n_c;      // channel blocks in total = B * n_dblk
+  int nwarps;       // warps per block = time sub-tiles per tile
+  int64_t tsteps;   // time steps per tile = nwarps * kWarpSteps
   int64_t n_t;      // time tiles
-  int64_t n_tiles;  // n_c * n_t
+  int ch_f, ch_b;   // channels per tile (forward, backward)
+  int64_t n_cg_f, n_cg_b;       // channel groups per batch row
+  int64_t n_c_f, n_c_b;         // channel groups in total (B * n_cg)
+  int64_t n_tiles_f, n_tiles_b; // n_t * n_c
   uint32_t tag;
-  // workspace byte offsets
-  size_t off_fhdr, off_fflags, off_bhdr, off_dlam, off_bflags;
+  // Workspace byte offsets. Records hold one entry per (time tile, channel):
+  // agg = (A, U) of the tile as one 64-bit word, pre = the state after it.
+  size_t off_fhdr, off_bhdr, off_dlam, off_k;
   size_t off_fagg, off_fpre, off_bagg, off_bpre, bytes;
 };
 
@@ -86,20 +96,21 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   p->D = D;
   p->io = io;
   p->c = c;
-  p->vec = (io == 0) ? 4 : 8;
-  p->tc = kTc;
-  p->dblk = (int)(D < kMaxDblk ? D : kMaxDblk);
-  p->nv = p->dblk / p->vec;
-  int64_t n_t = (L + kTargetTile - 1) / kTargetTile;
-  int64_t per = (L + n_t - 1) / n_t;                  // balanced tile length
-  int nt = (int)((per + p->tc - 1) / p->tc);
-  while (p->nv * nt < 32) ++nt;                         // at least one full warp
-  p->nt = nt;
-  p->ttile = (int64_t)nt * p->tc;
-  p->n_t = (L + p->ttile - 1) / p->ttile;
-  p->n_dblk = (D + p->dblk - 1) / p->dblk;
-  p->n_c = B * p->n_dblk;
-  p->n_tiles = p->n_c * p->n_t;
+  // Time tiling: as few tiles of up to kMaxWarps warps as cover L, balanced.
+  const int64_t max_steps = (int64_t)kMaxWarps * kWarpSteps;
+  const int64_t n_t0 = (L + max_steps - 1) / max_steps;
+  const int64_t per = (L + n_t0 - 1) / n_t0;
+  p->nwarps = (int)((per + kWarpSteps - 1) / kWarpSteps);
+  p->tsteps = (int64_t)p->nwarps * kWarpSteps;
+  p->n_t = (L + p->tsteps - 1) / p->tsteps;
+  p->ch_f = kNvl * fwd_vec(io);
+  p->ch_b = kNvl * bwd_vec(io);
+  p->n_cg_f = (D + p->ch_f - 1) / p->ch_f;
+  p->n_cg_b = (D + p->ch_b - 1) / p->ch_b;
+  p->n_c_f = B * p->n_cg_f;
+  p->n_c_b = B * p->n_cg_b;
+  p->n_tiles_f = p->n_t * p->n_c_f;
+  p->n_tiles_b = p->n_t * p->n_c_b;
   uint32_t h = 2166136261u;
   h = fnv1a(h, (uint64_t)B);
   h = fnv1a(h, (uint64_t)L);
@@ -109,23 +120,21 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   __builtin_memcpy(&cbits, &c, 4);
   h = fnv1a(h, cbits);
   p->tag = h | 1u;  // never 0, the value of a cleared header
+  const size_t rec = (size_t)p->n_t * (size_t)B * (size_t)D;  // one per (time tile, channel)
   size_t o = 0;
   p->off_fhdr = o;
   o = align_up(o + sizeof(FwdHeader), kAlign);
-  p->off_fflags = o;
-  o = align_up(o + 4 * (size_t)p->n_tiles, kAlign);
   p->off_bhdr = o;
   o = align_up(o + sizeof(BwdHeader), kAlign);
   p->off_dlam = o;
   o = align_up(o + 8 * (size_t)kStripes * (size_t)D, kAlign);
-  p->off_bflags = o;
-  o = align_up(o + 4 * (size_t)p->n_tiles, kAlign);
-  const size_t rec = (size_t)p->n_tiles * (size_t)p->dblk;
-  p->off_fagg = o;
+  p->off_k = o;
+  o = align_up(o + 4 * (size_t)D, kAlign);
+  p->off_fagg = o;  // forward records: agg then pre, filled together
   o = align_up(o + 8 * rec, kAlign);
   p->off_fpre = o;
   o = align_up(o + 4 * rec, kAlign);
-  p->off_bagg = o;
+  p->off_bagg = o;  // backward records
   o = align_up(o + 8 * rec, kAlign);
   p->off_bpre = o;
   o = align_up(o + 4 * rec, kAlign);
