@@ -173,6 +173,31 @@ BLR_API const char* blr_status_string(blr_status status);
 BLR_API const char* blr_last_error_string(void);
 
 /*
+ * Forward scan for callers that cannot allocate device memory (the paper has
+ * no counterpart; this is a deployment convenience). Code running inside CUDA
+ * stream capture, plugins whose host framework owns every device allocation,
+ * and serving loops that forbid allocator calls cannot provide the workspace
+ * blr_scan_fwd needs. This entry point computes exactly what blr_scan_fwd
+ * computes (same arguments except the workspace) on a scratch array that the
+ * library holds in device memory: 64 MiB, allocated on every GPU that loads
+ * the library and kept until the process exits. It never calls an allocator.
+ *  - Problems whose workspace (blr_workspace_bytes) exceeds 64 MiB return
+ *    BLR_ERR_UNSUPPORTED with nothing enqueued; use blr_scan_fwd for them.
+ *  - The first call on each device looks up the scratch array's device
+ *    address (cudaGetSymbolAddress); make that first call before any stream
+ *    capture that includes it.
+ *  - All calls on a device share the one scratch array, and each call reuses
+ *    whatever the last one left there after clearing what must start empty.
+ *    Calls that may overlap on the GPU (different streams without ordering
+ *    between them) race on it: serialise them.
+ *  - The scratch cannot be passed to blr_scan_bwd or blr_workspace_status:
+ *    this is a forward-only (inference) path.
+ */
+BLR_API blr_status blr_scan_fwd_noalloc(const blr_desc* desc, const void* x, const void* gate_logits,
+                                        const float* lambda, const float* h0, void* h,
+                                        float* h_last, blr_stream_t stream);
+
+/*
  * Diagnostic: runs one thread block that waits on a workspace flag nothing
  * sets, with the given bound in nanoseconds (at most 1e9), then records the
  * expired wait in the workspace. blr_workspace_status() then returns

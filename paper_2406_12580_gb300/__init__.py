@@ -25,7 +25,7 @@ from ._lib import (BLR_BF16, BLR_ERR_CUDA, BLR_ERR_INVALID_ARG, BLR_ERR_TIMEOUT,
 __all__ = [
     "BLR_F32", "BLR_BF16", "Desc", "BLRError", "blr_workspace_bytes", "blr_scan_fwd",
     "blr_scan_bwd", "blr_step", "blr_workspace_status", "blr_status_string",
-    "blr_selftest_wait_timeout", "BDLRUScan", "library_loaded",
+    "blr_selftest_wait_timeout", "blr_scan_fwd_noalloc", "BDLRUScan", "library_loaded",
 ]
 
 
@@ -129,6 +129,16 @@ def blr_selftest_wait_timeout(desc, ws, timeout_ns: int, stream=None):
     _check(load().blr_selftest_wait_timeout(ctypes.byref(desc), _ptr(ws, "ws"), ws.numel(),
                                             timeout_ns, _stream(stream)),
            "blr_selftest_wait_timeout")
+
+
+def blr_scan_fwd_noalloc(desc, x, gate_logits, lam, h0, h, h_last, stream=None):
+    """blr_scan_fwd on the library's static device scratch, for callers that
+    cannot allocate a workspace (see include/blr.h)."""
+    _check(load().blr_scan_fwd_noalloc(ctypes.byref(desc), _ptr(x, "x"),
+                                       _ptr(gate_logits, "gate_logits"), _ptr(lam, "lambda"),
+                                       _ptr(h0, "h0"), _ptr(h, "h"), _ptr(h_last, "h_last"),
+                                       _stream(stream)),
+           "blr_scan_fwd_noalloc")
 
 
 def blr_status_string(status: int) -> str:

@@ -43,6 +43,7 @@ SIGNATURES = {
     "blr_status_string": (ctypes.c_char_p, [_ST]),
     "blr_last_error_string": (ctypes.c_char_p, []),
     "blr_selftest_wait_timeout": (_ST, [_DESC_P, _VP, _SZ, ctypes.c_uint64, _VP]),
+    "blr_scan_fwd_noalloc": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
 }
 
 _lock = threading.Lock()

@@ -7,6 +7,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
+
 #include "blr.h"
 #include "blr_kernels.cuh"
 
@@ -304,3 +306,67 @@ const char* blr_status_string(blr_status status) {
 const char* blr_last_error_string(void) { return g_last_error; }
 
 }  // extern "C"
+
+// ----------------------------------------------------------------------------
+// Forward scan without a caller workspace (blr_scan_fwd_noalloc).
+//
+// Some callers cannot allocate device memory at the point where they run the
+// scan: code inside CUDA stream capture that may not add allocations, plugins
+// whose host framework owns every device allocation, or real-time serving
+// loops that forbid allocator calls. For them the forward scan can run on a
+// scratch array that lives in the library itself: a file-scope device array
+// of kNoAllocScratchBytes, present on every GPU that loads this library until
+// the process exits. The host never dereferences the array's name (in host
+// code it is only a stand-in for the device symbol); the device address comes
+// from cudaGetSymbolAddress, once per device.
+
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = (size_t)64 << 20;  // 64 MiB
+constexpr int kMaxDevices = 64;
+
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device (set up on the
+// first call on each device).
+blr_status noalloc_scratch(void** out) {
+  int dev = 0;
+  BLR_TRY(cuda_check(cudaGetDevice(&dev), "cudaGetDevice"));
+  if (dev < 0 || dev >= kMaxDevices)
+    return fail(BLR_ERR_UNSUPPORTED, "device index %d above the scratch table", dev);
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    BLR_TRY(cuda_check(cudaGetSymbolAddress(&p, g_noalloc_scratch),
+                       "cudaGetSymbolAddress of the static scratch"));
+    g_scratch_ptr[dev] = p;
+  }
+  *out = g_scratch_ptr[dev];
+  return BLR_OK;
+}
+
+}  // namespace
+
+extern "C" blr_status blr_scan_fwd_noalloc(const blr_desc* desc, const void* x,
+                                           const void* gate_logits, const float* lambda,
+                                           const float* h0, void* h, float* h_last,
+                                           blr_stream_t stream) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty || desc->L == 0)  // nothing that needs scratch: the ordinary path does it
+    return blr_scan_fwd(desc, x, gate_logits, lambda, h0, h, h_last, nullptr, 0, stream);
+  const size_t need_bytes = plan.bytes;
+  if (need_bytes > kNoAllocScratchBytes)
+    return fail(BLR_ERR_UNSUPPORTED,
+                "blr_scan_fwd_noalloc: this problem needs %zu bytes of scratch, above the %zu-byte "
+                "static scratch; use blr_scan_fwd with a caller workspace",
+                need_bytes, kNoAllocScratchBytes);
+  void* scratch = nullptr;
+  BLR_TRY(noalloc_scratch(&scratch));
+  return blr_scan_fwd(desc, x, gate_logits, lambda, h0, h, h_last, scratch, kNoAllocScratchBytes,
+                      stream);
+}
