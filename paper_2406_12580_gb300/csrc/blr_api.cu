@@ -9,6 +9,8 @@
 
 #include <mutex>
 
+#include <cudaTypedefs.h>
+
 #include "blr.h"
 #include "blr_kernels.cuh"
 
@@ -50,6 +52,10 @@ blr_status check_desc(const blr_desc* d, Plan* plan, bool* empty_bd) {
   if (d->B > (int64_t)1 << 40 || d->L > (int64_t)1 << 40 || d->D > (int64_t)1 << 24 ||
       (double)d->B * (double)d->L * (double)d->D > 1e18)
     return fail(BLR_ERR_UNSUPPORTED, "problem too large");
+  // TMA coordinates are 32-bit and tensor-map strides below 2^40 bytes.
+  if (d->B >= ((int64_t)1 << 31) || d->L >= ((int64_t)1 << 31) ||
+      (double)d->L * (double)d->D * 8.0 >= (double)((int64_t)1 << 40))
+    return fail(BLR_ERR_UNSUPPORTED, "problem too large for the tiled loads");
   blr::make_plan(d->B, d->L, d->D, (int)d->io, d->c, plan);
   if (plan->n_tiles_f >= ((int64_t)1 << 30) || plan->n_tiles_b >= ((int64_t)1 << 30))
     return fail(BLR_ERR_UNSUPPORTED, "too many tiles (%lld)", (long long)plan->n_tiles_b);
@@ -82,18 +88,87 @@ blr_status check_ws(const Plan& plan, const void* ws, size_t ws_bytes) {
 }
 
 // Persistent grid: as many blocks as fit on the device at once, at most one
-// per tile.
+// per tile. The per-device block count of each kernel (and its shared-memory
+// attribute) is set up once and cached: host time per call stays small.
+struct GridCacheEntry {
+  int dev;
+  const void* fn;
+  int threads;
+  size_t smem;
+  int blocks;  // blocks per SM x SMs
+};
+std::mutex g_grid_mutex;
+GridCacheEntry g_grid_cache[64];
+int g_grid_count = 0;
+
 template <typename K>
-blr_status persistent_grid(K kernel, int threads, int64_t n_tiles, unsigned* grid) {
-  int dev = 0, sms = 0, per_sm = 0;
+blr_status persistent_grid(K kernel, int threads, size_t smem, int64_t n_tiles, unsigned* grid) {
+  int dev = 0;
   BLR_TRY(cuda_check(cudaGetDevice(&dev), "cudaGetDevice"));
-  BLR_TRY(cuda_check(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev),
-                     "query SM count"));
-  BLR_TRY(cuda_check(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, 0),
-                     "query occupancy"));
-  int64_t g = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+  const void* fn = reinterpret_cast<const void*>(kernel);
+  int blocks = 0;
+  {
+    std::lock_guard<std::mutex> lock(g_grid_mutex);
+    for (int i = 0; i < g_grid_count; ++i) {
+      const GridCacheEntry& e = g_grid_cache[i];
+      if (e.dev == dev && e.fn == fn && e.threads == threads && e.smem == smem) blocks = e.blocks;
+    }
+    if (blocks == 0) {
+      int sms = 0, per_sm = 0;
+      BLR_TRY(cuda_check(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)smem),
+                         "set dynamic shared memory size"));
+      BLR_TRY(cuda_check(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev),
+                         "query SM count"));
+      BLR_TRY(cuda_check(
+          cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem),
+          "query occupancy"));
+      blocks = sms * (per_sm > 0 ? per_sm : 1);
+      if (g_grid_count < 64) g_grid_cache[g_grid_count++] = {dev, fn, threads, smem, blocks};
+    }
+  }
+  int64_t g = blocks;
   if (g > n_tiles) g = n_tiles;
   *grid = (unsigned)(g > 0 ? g : 1);
+  return BLR_OK;
+}
+
+// cuTensorMapEncodeTiled, through the runtime's driver entry point (the
+// library links only the CUDA runtime).
+blr_status tensor_map_encoder(PFN_cuTensorMapEncodeTiled_v12000* out) {
+  static std::mutex m;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::lock_guard<std::mutex> lock(m);
+  if (fn == nullptr) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    const cudaError_t e =
+        cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q);
+    if (e != cudaSuccess || q != cudaDriverEntryPointSuccess || ptr == nullptr)
+      return fail(BLR_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  *out = fn;
+  return BLR_OK;
+}
+
+// A 3-D tensor map over a row-major (B, L, cols) tensor seen as (cols, L, B),
+// boxes of 32 columns x `rows` steps x 1 batch row; out-of-range elements of
+// a box read as zero.
+blr_status make_tensor_map(CUtensorMap* map, const void* base, int io, int64_t cols, int64_t L,
+                           int64_t B, int64_t rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
+  BLR_TRY(tensor_map_encoder(&enc));
+  const cuuint64_t es = (io == BLR_F32) ? 4 : 2;
+  const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)L, (cuuint64_t)B};
+  const cuuint64_t strides[2] = {(cuuint64_t)cols * es, (cuuint64_t)cols * es * (cuuint64_t)L};
+  const cuuint32_t box[3] = {32u, (cuuint32_t)rows, 1u};
+  const cuuint32_t estr[3] = {1u, 1u, 1u};
+  const CUresult r = enc(map, io == BLR_F32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                         3, const_cast<void*>(base), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(BLR_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
   return BLR_OK;
 }
 
@@ -155,17 +230,26 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
   BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fagg,
                       plan.off_bagg - plan.off_fagg, reinterpret_cast<float*>(w + plan.off_k),
                       lambda, desc->D, desc->c, st));
-  blr::FwdArgs a{plan, x, gate_logits, h0, h, h_last, w};
+  blr::FwdArgs a;
+  BLR_TRY(make_tensor_map(&a.tm_x, x, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
+  BLR_TRY(make_tensor_map(&a.tm_gl, gate_logits, desc->io, 2 * desc->D, desc->L, desc->B, plan.tsteps));
+  a.p = plan;
+  a.h0 = h0;
+  a.h = h;
+  a.h_last = h_last;
+  a.ws = w;
   const int threads = plan.nwarps * 32;
   unsigned grid = 1;
   if (desc->io == BLR_F32) {
-    auto k = blr::scan_fwd_kernel<float, 4, blr::MathPrecise>;
-    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_f, &grid));
-    k<<<grid, threads, 0, st>>>(a);
+    auto k = blr::scan_fwd_kernel<float, blr::MathPrecise>;
+    const size_t smem = blr::ring_bytes<float, blr::fwd_stages<float>(), 3>();
+    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
+    k<<<grid, threads, smem, st>>>(a);
   } else {
-    auto k = blr::scan_fwd_kernel<__nv_bfloat16, 4, blr::MathFast>;
-    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_f, &grid));
-    k<<<grid, threads, 0, st>>>(a);
+    auto k = blr::scan_fwd_kernel<__nv_bfloat16, blr::MathFast>;
+    const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::fwd_stages<__nv_bfloat16>(), 3>();
+    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
+    k<<<grid, threads, smem, st>>>(a);
   }
   return cuda_check(cudaGetLastError(), "launch scan_fwd_kernel");
 }
@@ -207,17 +291,31 @@ blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_la
   BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, w + plan.off_bagg,
                       plan.bytes - plan.off_bagg, reinterpret_cast<float*>(w + plan.off_k), lambda,
                       desc->D, desc->c, st));
-  blr::BwdArgs a{plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda, dh0, w};
+  blr::BwdArgs a;
+  BLR_TRY(make_tensor_map(&a.tm_dh, dh, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
+  BLR_TRY(make_tensor_map(&a.tm_x, x, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
+  BLR_TRY(make_tensor_map(&a.tm_gl, gate_logits, desc->io, 2 * desc->D, desc->L, desc->B, plan.tsteps));
+  a.p = plan;
+  a.dh_last = dh_last;
+  a.lambda = lambda;
+  a.h0 = h0;
+  a.dx = dx;
+  a.dgl = dgate_logits;
+  a.dlambda = dlambda;
+  a.dh0 = dh0;
+  a.ws = w;
   const int threads = plan.nwarps * 32;
   unsigned grid = 1;
   if (desc->io == BLR_F32) {
-    auto k = blr::scan_bwd_kernel<float, 4, blr::MathPrecise>;
-    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_b, &grid));
-    k<<<grid, threads, 0, st>>>(a);
+    auto k = blr::scan_bwd_kernel<float, blr::MathPrecise>;
+    const size_t smem = blr::ring_bytes<float, blr::bwd_stages<float>(), 4>();
+    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
+    k<<<grid, threads, smem, st>>>(a);
   } else {
-    auto k = blr::scan_bwd_kernel<__nv_bfloat16, 4, blr::MathFast>;
-    BLR_TRY(persistent_grid(k, threads, plan.n_tiles_b, &grid));
-    k<<<grid, threads, 0, st>>>(a);
+    auto k = blr::scan_bwd_kernel<__nv_bfloat16, blr::MathFast>;
+    const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::bwd_stages<__nv_bfloat16>(), 4>();
+    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
+    k<<<grid, threads, smem, st>>>(a);
   }
   return cuda_check(cudaGetLastError(), "launch scan_bwd_kernel");
 }

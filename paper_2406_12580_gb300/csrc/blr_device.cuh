@@ -96,12 +96,15 @@ __device__ __forceinline__ void load_f32(const float* p, float (&v)[N]) {
 // 1 - alpha^2 = -E (2 + E), without the cancellation of 1 - alpha*alpha when
 // alpha is close to 1 (slow decays).
 //
-// Two precision policies. Float32 I/O (MathPrecise) uses CUDA's accurate expf,
-// correctly rounded reciprocal, division and square root, and a degree-8
-// Taylor polynomial for expm1. Bfloat16 I/O (MathFast), whose outputs carry 8
-// significant bits, uses the hardware approximations: sigmoid(z) =
-// (1 + tanh(z/2)) / 2 with tanh.approx (relative error below 2^-10.9),
-// ex2.approx, sqrt.approx and rsqrt.approx, and a degree-5 polynomial.
+// Two precision policies, both on the hardware's approximate units (whose
+// relative errors are at most about 2^-22 for ex2, rcp, rsqrt and sqrt, and
+// 2^-10.9 for tanh):
+//  * MathPrecise (float32 I/O): sigmoid(z) = 1 / (1 + 2^(-z log2 e)) with
+//    ex2.approx and rcp.approx (relative error below ~1.5e-6 for |z| <= 10),
+//    square roots through rsqrt.approx, and a degree-6 Taylor polynomial for
+//    expm1. End to end this keeps the float32 outputs near 1e-6 of float64.
+//  * MathFast (bfloat16 I/O, 8 significant bits out): sigmoid(z) =
+//    (1 + tanh(z/2)) / 2 with tanh.approx, and a degree-4 polynomial.
 
 __device__ __forceinline__ float tanh_approx(float x) {
   float y;
@@ -136,34 +139,70 @@ __device__ __forceinline__ float expm1_taylor(float l) {
   return p * l;
 }
 
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// sqrt(q) and 1 / sqrt(q) for q >= 0 (0 and 0 at q = 0).
+__device__ __forceinline__ void sqrt_pair(float q, float& n, float& inv_n) {
+  const float rs = rsqrt_approx(q);
+  const bool pos = q > 0.0f;
+  n = pos ? q * rs : 0.0f;
+  inv_n = pos ? rs : 0.0f;
+}
+
 struct MathPrecise {
   static __device__ __forceinline__ float sigmoid(float z) {
-    return __frcp_rn(1.0f + expf(-z));
+    return rcp_approx(1.0f + ex2_approx(-1.4426950408889634f * z));
   }
-  // e^l - 1 for l <= 0: the degree-8 series (truncation below l^8/9! < 5e-11
-  // relative for l > -0.25) near zero, where decays usually live
-  // (|l| <= softplus(Lambda) <= 0.11 for base decays in [0.9, 1)); beyond it
-  // e^l < 0.78 and e^l - 1 loses nothing to cancellation.
-  static __device__ __forceinline__ float expm1_nonpos(float l) {
-    if (l > -0.25f) return expm1_taylor<8>(l);
-    return expf(l) - 1.0f;
+  // e^l - 1 for -0.25 < l <= 0: the degree-6 series (truncation below
+  // l^6/7! < 5e-8 relative). Decays usually live there: |l| <= softplus(Lambda)
+  // <= 0.11 for base decays in [0.9, 1).
+  static __device__ __forceinline__ float expm1_poly(float l) { return expm1_taylor<6>(l); }
+  // Any l <= 0: beyond the series' range e^l < 0.78 and e^l - 1 loses
+  // nothing to cancellation.
+  static __device__ __forceinline__ float expm1_any(float l) {
+    if (l > -0.25f) return expm1_taylor<6>(l);
+    return ex2_approx(l * 1.4426950408889634f) - 1.0f;
   }
-  static __device__ __forceinline__ float sqrt(float q) { return __fsqrt_rn(q); }
-  static __device__ __forceinline__ float div(float a, float b) { return __fdiv_rn(a, b); }
+  static __device__ __forceinline__ float sqrt(float q) {
+    float n, inv_n;
+    sqrt_pair(q, n, inv_n);
+    return n;
+  }
+  // beta = sqrt(q) i, u = beta x and c2 = alpha u / q (= alpha i x / n).
+  static __device__ __forceinline__ void norm_terms(float q, float i, float x, float alpha,
+                                                    float& beta, float& u, float& c2) {
+    float n, inv_n;
+    sqrt_pair(q, n, inv_n);
+    beta = n * i;
+    u = beta * x;
+    c2 = alpha * u * (inv_n * inv_n);
+  }
 };
 
 struct MathFast {
   static __device__ __forceinline__ float sigmoid(float z) {
     return fmaf(0.5f, tanh_approx(0.5f * z), 0.5f);
   }
-  // Degree-5 series near zero (truncation below l^5/6! < 1.4e-6 relative for
-  // l > -0.25), ex2.approx beyond.
-  static __device__ __forceinline__ float expm1_nonpos(float l) {
-    if (l > -0.25f) return expm1_taylor<5>(l);
+  // Degree-4 series for -0.25 < l <= 0 (truncation below l^4/5! < 3.3e-5
+  // relative), ex2.approx beyond.
+  static __device__ __forceinline__ float expm1_poly(float l) { return expm1_taylor<4>(l); }
+  static __device__ __forceinline__ float expm1_any(float l) {
+    if (l > -0.25f) return expm1_taylor<4>(l);
     return ex2_approx(l * 1.4426950408889634f) - 1.0f;
   }
   static __device__ __forceinline__ float sqrt(float q) { return sqrt_approx(q); }
-  static __device__ __forceinline__ float div(float a, float b) { return __fdividef(a, b); }
+  static __device__ __forceinline__ void norm_terms(float q, float i, float x, float alpha,
+                                                    float& beta, float& u, float& c2) {
+    float n, inv_n;
+    sqrt_pair(q, n, inv_n);
+    beta = n * i;
+    u = beta * x;
+    c2 = alpha * u * (inv_n * inv_n);
+  }
 };
 
 // k = -c softplus(Lambda), softplus(z) = max(z, 0) + log1p(exp(-|z|)), accurate.
@@ -243,6 +282,66 @@ __device__ __noinline__ bool wait_word(const uint32_t* flag, uint32_t* err, uint
       }
     }
   }
+}
+
+// ------------------------------------------------------------- TMA and mbarrier
+//
+// Tiles of the inputs are moved into shared memory by the tensor memory
+// accelerator (cp.async.bulk.tensor, 3-D boxes of 32 channels x tile steps x
+// one batch row) and counted on an mbarrier per pipeline stage.
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Waits for the stage's loads to land. Bounded: after the limit the block
+// records kErrTimeout and goes on with whatever the stage holds.
+__device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  if (mbar_try_wait(bar, parity)) return;
+  const uint64_t start = global_timer_ns();
+  for (uint32_t iter = 0;; ++iter) {
+    if (mbar_try_wait(bar, parity)) return;
+    if ((iter & 15u) == 15u && (global_timer_ns() - start > kWaitTimeoutNs || iter > kMaxWaitIters)) {
+      atomicOr(err, kErrTimeout);
+      return;
+    }
+  }
+}
+
+// One 3-D tile load: box at (c0, c1, c2) of the tensor map into shared memory.
+__device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, uint64_t* bar, int c0,
+                                            int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_addr(dst)),
+      "l"(tmap), "r"(c0), "r"(c1), "r"(c2), "r"(smem_addr(bar))
+      : "memory");
 }
 
 }  // namespace blr

@@ -20,6 +20,7 @@
 // one after warp 0's part are the only block-wide synchronisation per tile.
 #pragma once
 
+#include <cuda.h>
 #include <limits.h>
 
 #include "blr_device.cuh"
@@ -28,10 +29,13 @@ namespace blr {
 
 constexpr unsigned kFull = 0xffffffffu;
 
+// Inputs reach the scan kernels through TMA tensor maps over 3-D views
+// (channels, time, batch) of the row-major tensors: x and dh as (D, L, B),
+// gate_logits as (2D, L, B).
 struct FwdArgs {
+  CUtensorMap tm_x;
+  CUtensorMap tm_gl;
   Plan p;
-  const void* x;
-  const void* gl;
   const float* h0;
   void* h;
   float* h_last;
@@ -39,11 +43,11 @@ struct FwdArgs {
 };
 
 struct BwdArgs {
+  CUtensorMap tm_dh;
+  CUtensorMap tm_x;
+  CUtensorMap tm_gl;
   Plan p;
-  const void* dh;
   const float* dh_last;
-  const void* x;
-  const void* gl;
   const float* lambda;
   const float* h0;
   void* dx;
@@ -52,6 +56,34 @@ struct BwdArgs {
   float* dh0;
   unsigned char* ws;
 };
+
+// Shared-memory ring of the scan kernels: STAGES stages of NB boxes, each box
+// kMaxTile rows x 32 channels, then one mbarrier per stage.
+constexpr int kMaxTile = kMaxWarps * kWarpSteps;
+template <typename T>
+__host__ __device__ constexpr uint32_t box_bytes() {
+  return (uint32_t)(kMaxTile * 32 * sizeof(T));
+}
+template <typename T, int STAGES, int NB>
+__host__ __device__ constexpr size_t ring_bytes() {  // + slack to align the ring to 1 KiB
+  return (size_t)STAGES * NB * box_bytes<T>() + (size_t)STAGES * sizeof(uint64_t) + 1024;
+}
+
+// The ring's base: the dynamic shared memory rounded up to 1 KiB.
+__device__ __forceinline__ unsigned char* ring_base(unsigned char* dyn) {
+  const uint32_t a = smem_addr(dyn);
+  return dyn + (((a + 1023u) & ~1023u) - a);
+}
+// Stages per block, sized so that four forward (three backward) blocks fit an
+// SM's shared memory.
+template <typename T>
+__host__ __device__ constexpr int fwd_stages() {
+  return sizeof(T) == 4 ? 2 : 4;
+}
+template <typename T>
+__host__ __device__ constexpr int bwd_stages() {
+  return sizeof(T) == 4 ? 2 : 3;
+}
 
 struct StepArgs {
   int64_t B, D;
@@ -84,12 +116,12 @@ __global__ void prep_kernel(uint32_t* zero, int64_t zero_words, uint4* fill, int
 // Lane layout: lane = tcl * kNvl + cv. The kNtl lanes with the same cv hold
 // consecutive chunks in time of the same channels.
 
-// Turns each lane's chunk map (A, U) into the exclusive prefix map of the
-// chunks before it in the warp (ea, eu), and returns the warp's map (ta, tu).
+// Turns each lane's chunk map (A, U) into the inclusive prefix map of the
+// chunks up to it (A, U; the last time lane then holds the warp's map) and the
+// exclusive one (ea, eu).
 template <int V>
-__device__ __forceinline__ void warp_prefix(float (&A)[V], float (&U)[V], int tcl, int cv,
-                                            float (&ea)[V], float (&eu)[V], float (&ta)[V],
-                                            float (&tu)[V]) {
+__device__ __forceinline__ void warp_prefix(float (&A)[V], float (&U)[V], int tcl,
+                                            float (&ea)[V], float (&eu)[V]) {
 #pragma unroll
   for (int off = 1; off < kNtl; off <<= 1) {
 #pragma unroll
@@ -110,18 +142,16 @@ __device__ __forceinline__ void warp_prefix(float (&A)[V], float (&U)[V], int tc
       ea[v] = 1.0f;
       eu[v] = 0.0f;
     }
-    ta[v] = __shfl_sync(kFull, A[v], (kNtl - 1) * kNvl + cv);
-    tu[v] = __shfl_sync(kFull, U[v], (kNtl - 1) * kNvl + cv);
   }
 }
 
-// The same from the end of the warp's time range: (sa, sw) maps the value
-// entering after the warp's last step to the value entering after this
-// lane's chunk; (ta, tw) is the warp's map.
+// The same from the end of the warp's time range: (A, W) becomes the map from
+// the value entering after the warp's last step to the value at this lane's
+// chunk start (the first time lane then holds the warp's map), and (sa, sw)
+// the map to the value entering after this lane's chunk.
 template <int V>
-__device__ __forceinline__ void warp_suffix(float (&A)[V], float (&W)[V], int tcl, int cv,
-                                            float (&sa)[V], float (&sw)[V], float (&ta)[V],
-                                            float (&tw)[V]) {
+__device__ __forceinline__ void warp_suffix(float (&A)[V], float (&W)[V], int tcl,
+                                            float (&sa)[V], float (&sw)[V]) {
 #pragma unroll
   for (int off = 1; off < kNtl; off <<= 1) {
 #pragma unroll
@@ -142,8 +172,6 @@ __device__ __forceinline__ void warp_suffix(float (&A)[V], float (&W)[V], int tc
       sa[v] = 1.0f;
       sw[v] = 0.0f;
     }
-    ta[v] = __shfl_sync(kFull, A[v], cv);
-    tw[v] = __shfl_sync(kFull, W[v], cv);
   }
 }
 
@@ -195,10 +223,10 @@ __device__ __forceinline__ float lookback(const unsigned long long* agg, const u
 
 // ------------------------------------------------------------ tile tickets
 //
-// A ticket is decoded once, by the lane that draws it, into the tile's
-// position; blocks keep the decoded tiles in a three-slot ring: the tile being
-// finished, the next one (whose inputs are already being loaded) and the one
-// after (drawn during the current tile).
+// A ticket is decoded once, by the thread that draws it, into the tile's
+// position. Blocks keep decoded tiles in a ring: the tile being finished, the
+// tiles whose inputs are in flight in the shared-memory stages, and the next
+// one drawn.
 
 struct TileCoord {
   int64_t tile;   // the ticket; >= the tile count means no tile
@@ -223,128 +251,206 @@ __device__ __forceinline__ TileCoord decode_tile(int64_t tile, int64_t n_tiles, 
   return c;
 }
 
-// ---------------------------------------------------------------- forward scan
+// ---------------------------------------------------------- gate arithmetic
+//
+// e^l - 1 for l = k r <= 0: the polynomial alone when |k| <= kPolyLimit (then
+// |l| <= kPolyLimit for every r in [0, 1]), else the general form.
+constexpr float kPolyLimit = 0.25f;
 
-template <typename T, int VEC, class M>
-__global__ void __launch_bounds__(kMaxWarps * 32, 3) scan_fwd_kernel(const FwdArgs a) {
-  using IO = Io<T, VEC>;
-  using Raw = typename IO::Raw;
-  constexpr int CH = kNvl * VEC;
-  static_assert(CH == 32, "warp 0 handles one channel per lane");
-  const Plan& p = a.p;
+template <class M, bool POLY>
+__device__ __forceinline__ float gate_expm1(float l) {
+  if (POLY) return M::expm1_poly(l);
+  return M::expm1_any(l);
+}
 
-  __shared__ float2 s_wmap[2][kMaxWarps][CH];  // warp maps, then warp prefix maps
-  __shared__ float s_carry[2][CH];
-  __shared__ TileCoord s_tc[3];
-
-  FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
-  unsigned long long* agg = reinterpret_cast<unsigned long long*>(a.ws + p.off_fagg);
-  uint32_t* pre = reinterpret_cast<uint32_t*>(a.ws + p.off_fpre);
-  const float* kd = reinterpret_cast<const float*>(a.ws + p.off_k);
-  const T* x = static_cast<const T*>(a.x);
-  const T* gl = static_cast<const T*>(a.gl);
-  T* h = static_cast<T*>(a.h);
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int cv = lane % kNvl, tcl = lane / kNvl;
-  const int64_t BD = p.B * p.D;
-  const int64_t lane_t = (int64_t)warp * kWarpSteps + tcl * kTc;  // first step within a tile
-
-  auto decode = [&](uint32_t t) {
-    return decode_tile((int64_t)t, p.n_tiles_f, p.n_c_f, p.n_cg_f, CH, p.n_t, false);
-  };
-  const bool drawer = threadIdx.x == blockDim.x - 1;  // draws the tickets
-  if (drawer) {
-    s_tc[0] = decode(atomicAdd(&fh->ticket, 1u));
-    s_tc[1] = decode(atomicAdd(&fh->ticket, 1u));
-  }
-  __syncthreads();
-
-  // The raw inputs of the next tile, in flight while the current one finishes.
-  Raw nx[kTc], nr[kTc], ni[kTc];
-  float nk[VEC];
-  auto fetch = [&](const TileCoord& c) {
-    const int64_t d0 = c.dbase + cv * VEC;
-    const int64_t t0 = c.tt * p.tsteps + lane_t;
+// One lane's rows of a box in a stage: rows row0 .. row0 + kTc - 1, channels
+// cv*VEC .. cv*VEC + VEC - 1 (box rows are 32 channels wide).
+template <class IO>
+__device__ __forceinline__ void lds_rows(const unsigned char* box, int row0, int cv,
+                                         typename IO::Raw (&r)[kTc]) {
+  using T = typename IO::T;
+  const T* base = reinterpret_cast<const T*>(box) + row0 * 32 + cv * IO::VEC;
 #pragma unroll
-    for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
-    if (d0 < p.D) {
-      load_f32<VEC>(kd + d0, nk);
-      const T* px = x + (c.b * p.L + t0) * p.D + d0;
-      const T* pg = gl + (c.b * p.L + t0) * 2 * p.D + d0;
+  for (int s = 0; s < kTc; ++s) r[s] = *reinterpret_cast<const typename IO::Raw*>(base + s * 32);
+}
+
+// Forward gates of a lane's chunk: alpha and u = sqrt(1 - alpha^2) i x per
+// element; FULL when every element is inside the sequence and the channels,
+// else elements outside become the identity map (alpha = 1, u = 0).
+template <class IO, class M, bool FULL>
+__device__ __forceinline__ void fwd_chunk(const float (&k)[4],
+                                          const typename IO::Raw (&rx)[kTc],
+                                          const typename IO::Raw (&rr)[kTc],
+                                          const typename IO::Raw (&ri)[kTc], int valid,
+                                          float (&al)[kTc][4], float (&u)[kTc][4]) {
+  float xv[kTc][4], rv[kTc][4], iv[kTc][4];
+#pragma unroll
+  for (int s = 0; s < kTc; ++s) {
+    IO::unpack(rx[s], xv[s]);
+    IO::unpack(rr[s], rv[s]);
+    IO::unpack(ri[s], iv[s]);
+  }
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    if (k[v] >= -kPolyLimit) {
 #pragma unroll
       for (int s = 0; s < kTc; ++s) {
-        if (t0 + s < p.L) {
-          nx[s] = IO::load_raw(px + s * p.D);
-          nr[s] = IO::load_raw(pg + s * 2 * p.D);
-          ni[s] = IO::load_raw(pg + s * 2 * p.D + p.D);
-        }
+        const float r = M::sigmoid(rv[s][v]);
+        const float i = M::sigmoid(iv[s][v]);
+        const float e = gate_expm1<M, true>(k[v] * r);
+        al[s][v] = 1.0f + e;
+        u[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
+      }
+    } else {
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        const float r = M::sigmoid(rv[s][v]);
+        const float i = M::sigmoid(iv[s][v]);
+        const float e = gate_expm1<M, false>(k[v] * r);
+        al[s][v] = 1.0f + e;
+        u[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
       }
     }
-  };
-  if (s_tc[0].tile < p.n_tiles_f) fetch(s_tc[0]);
-
-  for (int it = 0;; ++it) {
-    const int buf = it & 1;
-    const TileCoord tc = s_tc[it % 3];
-    if (tc.tile >= p.n_tiles_f) break;
-    const int64_t d0 = tc.dbase + cv * VEC;
-    const bool ch_ok = d0 < p.D;
-    const int64_t t0 = tc.tt * p.tsteps + lane_t;
-    // the ticket after next: drawn now, decoded before the barrier
-    const uint32_t ticket = drawer ? atomicAdd(&fh->ticket, 1u) : 0u;
-
-    // 1. gates and chunk map from the raw registers
-    float k[VEC];
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) k[v] = nk[v];
-    float al[kTc][VEC], u[kTc][VEC];
+  }
+  if (!FULL) {
 #pragma unroll
     for (int s = 0; s < kTc; ++s) {
-      const bool ok = ch_ok && t0 + s < p.L;
-      float xv[VEC], rv[VEC], iv[VEC];
-      IO::unpack(nx[s], xv);
-      IO::unpack(nr[s], rv);
-      IO::unpack(ni[s], iv);
+      if (s >= valid) {
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        if (ok) {
-          const float r = M::sigmoid(rv[v]);
-          const float i = M::sigmoid(iv[v]);
-          const float e = M::expm1_nonpos(k[v] * r);
-          al[s][v] = 1.0f + e;
-          u[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[v];
-        } else {  // outside the sequence or the channels: the identity map
+        for (int v = 0; v < 4; ++v) {
           al[s][v] = 1.0f;
           u[s][v] = 0.0f;
         }
       }
     }
-    // the next tile's inputs start moving now
+  }
+}
+
+// ---------------------------------------------------------------- forward scan
+
+template <typename T, class M>
+__global__ void __launch_bounds__(kMaxWarps * 32, 4)
+    scan_fwd_kernel(const __grid_constant__ FwdArgs a) {
+  using IO = Io<T, 4>;
+  using Raw = typename IO::Raw;
+  constexpr int VEC = 4;
+  constexpr int CH = kNvl * VEC;
+  constexpr int S = fwd_stages<T>();
+  constexpr int NB = 3;  // boxes per stage: x, rho, iota
+  constexpr int RING = S + 2;
+  static_assert(CH == 32, "warp 0 handles one channel per lane");
+  const Plan& p = a.p;
+
+  extern __shared__ __align__(1024) unsigned char dyn_smem[];
+  unsigned char* smem = ring_base(dyn_smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * NB * box_bytes<T>());
+  __shared__ float2 s_wmap[2][kMaxWarps][CH];  // warp maps, then warp prefix maps
+  __shared__ float s_carry[2][CH];
+  __shared__ TileCoord s_tc[RING];
+
+  FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
+  unsigned long long* agg = reinterpret_cast<unsigned long long*>(a.ws + p.off_fagg);
+  uint32_t* pre = reinterpret_cast<uint32_t*>(a.ws + p.off_fpre);
+  const float* kd = reinterpret_cast<const float*>(a.ws + p.off_k);
+  T* h = static_cast<T*>(a.h);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cv = lane % kNvl, tcl = lane / kNvl;
+  const int64_t BD = p.B * p.D;
+  const int row0 = warp * kWarpSteps + tcl * kTc;  // this lane's first row in a tile
+  const uint32_t box_tx = (uint32_t)p.tsteps * CH * sizeof(T);
+  const bool drawer = threadIdx.x == blockDim.x - 1;  // draws the tickets
+
+  auto decode = [&](uint32_t t) {
+    return decode_tile((int64_t)t, p.n_tiles_f, p.n_c_f, p.n_cg_f, CH, p.n_t, false);
+  };
+  auto issue = [&](int stage, const TileCoord& c) {  // one thread: the tile's boxes into a stage
+    unsigned char* dst = smem + (size_t)stage * NB * box_bytes<T>();
+    const int t = (int)(c.tt * p.tsteps), d = (int)c.dbase, bb = (int)c.b;
+    mbar_arrive_expect_tx(&bars[stage], NB * box_tx);
+    tma_load_3d(dst, &a.tm_x, &bars[stage], d, t, bb);
+    tma_load_3d(dst + box_bytes<T>(), &a.tm_gl, &bars[stage], d, t, bb);
+    tma_load_3d(dst + 2 * box_bytes<T>(), &a.tm_gl, &bars[stage], (int)p.D + d, t, bb);
+  };
+
+  if (threadIdx.x == 0) {
+    for (int j = 0; j < S; ++j) mbar_init(&bars[j], 1);
+    fence_mbar_init();
+  }
+  if (drawer) {
+    for (int j = 0; j <= S; ++j) s_tc[j] = decode(atomicAdd(&fh->ticket, 1u));
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int j = 0; j < S; ++j)
+      if (s_tc[j].tile < p.n_tiles_f) issue(j, s_tc[j]);
+  }
+  float nk[VEC];  // k of the next tile's channels
+  {
+    const TileCoord& c = s_tc[0];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+    if (c.tile < p.n_tiles_f && c.dbase + cv * VEC < p.D) load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
+  }
+
+  for (int it = 0;; ++it) {
+    const int stage = it % S;
+    const int buf = it & 1;
+    const TileCoord tc = s_tc[it % RING];
+    if (tc.tile >= p.n_tiles_f) break;
+    const int64_t d0 = tc.dbase + cv * VEC;
+    const bool ch_ok = d0 < p.D;
+    const int64_t t0 = tc.tt * p.tsteps + row0;
+    int64_t left = ch_ok ? p.L - t0 : 0;
+    const int valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
+    const uint32_t ticket = drawer ? atomicAdd(&fh->ticket, 1u) : 0u;  // decoded before B1
+    float k[VEC];
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) k[v] = nk[v];
     {
-      const TileCoord nc = s_tc[(it + 1) % 3];
-      if (nc.tile < p.n_tiles_f) fetch(nc);
+      const TileCoord& c = s_tc[(it + 1) % RING];
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+      if (c.tile < p.n_tiles_f && c.dbase + cv * VEC < p.D)
+        load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
     }
+
+    // 1. the stage's rows of this lane, gates, chunk map
+    mbar_wait(&bars[stage], (uint32_t)(it / S) & 1u, &fh->err);
+    const unsigned char* sb = smem + (size_t)stage * NB * box_bytes<T>();
+    Raw rx[kTc], rr[kTc], ri[kTc];
+    lds_rows<IO>(sb, row0, cv, rx);
+    lds_rows<IO>(sb + box_bytes<T>(), row0, cv, rr);
+    lds_rows<IO>(sb + 2 * box_bytes<T>(), row0, cv, ri);
+    float al[kTc][VEC], u[kTc][VEC];
+    if (valid == kTc)
+      fwd_chunk<IO, M, true>(k, rx, rr, ri, valid, al, u);
+    else
+      fwd_chunk<IO, M, false>(k, rx, rr, ri, valid, al, u);
     float A[VEC], U[VEC];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) {
-      A[v] = 1.0f;
-      U[v] = 0.0f;
+      A[v] = al[0][v];
+      U[v] = u[0][v];
 #pragma unroll
-      for (int s = 0; s < kTc; ++s) {
+      for (int s = 1; s < kTc; ++s) {
         U[v] = fmaf(al[s][v], U[v], u[s][v]);
         A[v] *= al[s][v];
       }
     }
     // 2. warp prefix maps
-    float ea[VEC], eu[VEC], wa[VEC], wu[VEC];
-    warp_prefix<VEC>(A, U, tcl, cv, ea, eu, wa, wu);
+    float ea[VEC], eu[VEC];
+    warp_prefix<VEC>(A, U, tcl, ea, eu);
     if (tcl == kNtl - 1) {
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) s_wmap[buf][warp][cv * VEC + v] = make_float2(wa[v], wu[v]);
+      for (int v = 0; v < VEC; ++v) s_wmap[buf][warp][cv * VEC + v] = make_float2(A[v], U[v]);
     }
-    if (drawer) s_tc[(it + 2) % 3] = decode(ticket);
-    __syncthreads();
+    if (drawer) s_tc[(it + S + 1) % RING] = decode(ticket);
+    __syncthreads();  // the stage is read: refill it with the tile S ahead
+    if (threadIdx.x == 0) {
+      const TileCoord& c = s_tc[(it + S) % RING];
+      if (c.tile < p.n_tiles_f) issue(stage, c);
+    }
 
     // 3. warp 0, one lane per channel: tile map, look-back, tile prefix
     if (warp == 0) {
@@ -391,7 +497,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3) scan_fwd_kernel(const FwdAr
           hs[v] = fmaf(al[s][v], hs[v], u[s][v]);
           out[v] = hs[v];
         }
-        if (t0 + s < p.L) IO::store(ph + s * p.D, out);
+        if (s < valid) IO::store(ph + s * p.D, out);
       }
     }
   }
@@ -420,21 +526,105 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3) scan_fwd_kernel(const FwdAr
 //   dLambda += dl (-c r) sigmoid(Lambda)      (summed over b, t)
 // h_{t-1} is rebuilt from the forward's per-tile carries, not read from h.
 
-template <typename T, int VEC, class M>
-__global__ void __launch_bounds__(kMaxWarps * 32, sizeof(T) == 4 ? 2 : 3)
-    scan_bwd_kernel(const BwdArgs a) {
-  using IO = Io<T, VEC>;
+// Backward first pass over a lane's chunk: keeps E = expm1(l), r, i (and
+// x, dh) per element and folds the chunk's maps (A, U) forwards and W
+// backwards; elements outside the sequence or the channels are the identity.
+template <class IO, class M, bool FULL>
+__device__ __forceinline__ void bwd_chunk(const float (&k)[4], const typename IO::Raw (&rg)[kTc],
+                                          const typename IO::Raw (&rx)[kTc],
+                                          const typename IO::Raw (&rr)[kTc],
+                                          const typename IO::Raw (&ri)[kTc], int valid,
+                                          float (&gv)[kTc][4], float (&xv)[kTc][4],
+                                          float (&ev)[kTc][4], float (&rv)[kTc][4],
+                                          float (&iv)[kTc][4], float (&A)[4], float (&U)[4],
+                                          float (&W)[4]) {
+#pragma unroll
+  for (int s = 0; s < kTc; ++s) {
+    IO::unpack(rg[s], gv[s]);
+    IO::unpack(rx[s], xv[s]);
+    IO::unpack(rr[s], rv[s]);
+    IO::unpack(ri[s], iv[s]);
+  }
+  float uu[kTc][4];
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    if (k[v] >= -kPolyLimit) {
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        const float r = M::sigmoid(rv[s][v]);
+        const float i = M::sigmoid(iv[s][v]);
+        const float e = gate_expm1<M, true>(k[v] * r);
+        uu[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
+        rv[s][v] = r;
+        iv[s][v] = i;
+        ev[s][v] = e;
+      }
+    } else {
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        const float r = M::sigmoid(rv[s][v]);
+        const float i = M::sigmoid(iv[s][v]);
+        const float e = gate_expm1<M, false>(k[v] * r);
+        uu[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
+        rv[s][v] = r;
+        iv[s][v] = i;
+        ev[s][v] = e;
+      }
+    }
+  }
+  if (!FULL) {
+#pragma unroll
+    for (int s = 0; s < kTc; ++s) {
+      if (s >= valid) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          ev[s][v] = 0.0f;
+          rv[s][v] = 0.0f;
+          iv[s][v] = 0.0f;
+          gv[s][v] = 0.0f;
+          xv[s][v] = 0.0f;
+          uu[s][v] = 0.0f;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    A[v] = 1.0f;
+    U[v] = 0.0f;
+    W[v] = 0.0f;
+#pragma unroll
+    for (int s = 0; s < kTc; ++s) {
+      const float alpha = 1.0f + ev[s][v];
+      U[v] = fmaf(alpha, U[v], uu[s][v]);
+      A[v] *= alpha;                      // prod of alpha up to and including s
+      W[v] = fmaf(A[v], gv[s][v], W[v]);  // w at the chunk start from a zero carry
+    }
+  }
+}
+
+template <typename T, class M>
+__global__ void __launch_bounds__(kMaxWarps * 32, 3)
+    scan_bwd_kernel(const __grid_constant__ BwdArgs a) {
+  using IO = Io<T, 4>;
   using Raw = typename IO::Raw;
+  constexpr int VEC = 4;
   constexpr int CH = kNvl * VEC;
+  constexpr int S = bwd_stages<T>();
+  constexpr int NB = 4;  // boxes per stage: dh, x, rho, iota
+  constexpr int RING = S + 2;
   static_assert(CH == 32, "warp 0 handles one channel per lane");
   const Plan& p = a.p;
 
+  extern __shared__ __align__(1024) unsigned char dyn_smem[];
+  unsigned char* smem = ring_base(dyn_smem);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * NB * box_bytes<T>());
   __shared__ float s_wa[2][kMaxWarps][CH];   // warp prod alpha -> warp prefix map A
   __shared__ float s_wu[2][kMaxWarps][CH];   // warp U          -> warp prefix map U
   __shared__ float s_ww[2][kMaxWarps][CH];   // warp W          -> warp suffix map W
   __shared__ float s_ws[2][kMaxWarps][CH];   //                 -> warp suffix map A
   __shared__ float s_hc[2][CH], s_wc[2][CH];
-  __shared__ TileCoord s_tc[3];
+  __shared__ TileCoord s_tc[RING];
   __shared__ int s_flag;
 
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
@@ -444,135 +634,116 @@ __global__ void __launch_bounds__(kMaxWarps * 32, sizeof(T) == 4 ? 2 : 3)
   const float* fpre = reinterpret_cast<const float*>(a.ws + p.off_fpre);
   const float* kd = reinterpret_cast<const float*>(a.ws + p.off_k);
   double* dlam_acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
-  const T* x = static_cast<const T*>(a.x);
-  const T* gl = static_cast<const T*>(a.gl);
-  const T* dh = static_cast<const T*>(a.dh);
   T* dx = static_cast<T*>(a.dx);
   T* dgl = static_cast<T*>(a.dgl);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int cv = lane % kNvl, tcl = lane / kNvl;
   const int64_t BD = p.B * p.D;
-  const int64_t lane_t = (int64_t)warp * kWarpSteps + tcl * kTc;
+  const int row0 = warp * kWarpSteps + tcl * kTc;
+  const uint32_t box_tx = (uint32_t)p.tsteps * CH * sizeof(T);
+  const bool drawer = threadIdx.x == blockDim.x - 1;
 
   auto decode = [&](uint32_t t) {
     return decode_tile((int64_t)t, p.n_tiles_b, p.n_c_b, p.n_cg_b, CH, p.n_t, true);
   };
-  const bool drawer = threadIdx.x == blockDim.x - 1;  // draws the tickets
+  auto issue = [&](int stage, const TileCoord& c) {
+    unsigned char* dst = smem + (size_t)stage * NB * box_bytes<T>();
+    const int t = (int)(c.tt * p.tsteps), d = (int)c.dbase, bb = (int)c.b;
+    mbar_arrive_expect_tx(&bars[stage], NB * box_tx);
+    tma_load_3d(dst, &a.tm_dh, &bars[stage], d, t, bb);
+    tma_load_3d(dst + box_bytes<T>(), &a.tm_x, &bars[stage], d, t, bb);
+    tma_load_3d(dst + 2 * box_bytes<T>(), &a.tm_gl, &bars[stage], d, t, bb);
+    tma_load_3d(dst + 3 * box_bytes<T>(), &a.tm_gl, &bars[stage], (int)p.D + d, t, bb);
+  };
+
+  if (threadIdx.x == 0) {
+    for (int j = 0; j < S; ++j) mbar_init(&bars[j], 1);
+    fence_mbar_init();
+  }
   if (drawer) {
     const bool ok = __ldcg(&fh->tag) == p.tag && __ldcg(&fh->complete) == 1u;
     if (!ok) atomicOr(&fh->err, kErrWorkspace);
     s_flag = ok;
-    if (ok) {
-      s_tc[0] = decode(atomicAdd(&bh->ticket, 1u));
-      s_tc[1] = decode(atomicAdd(&bh->ticket, 1u));
-    }
+    if (ok)
+      for (int j = 0; j <= S; ++j) s_tc[j] = decode(atomicAdd(&bh->ticket, 1u));
   }
   __syncthreads();
   if (!s_flag) return;  // no forward carries for this problem: write nothing
-
-  Raw ng[kTc], nx[kTc], nr[kTc], ni[kTc];
+  if (threadIdx.x == 0) {
+    for (int j = 0; j < S; ++j)
+      if (s_tc[j].tile < p.n_tiles_b) issue(j, s_tc[j]);
+  }
   float nk[VEC];
-  auto fetch = [&](const TileCoord& c) {
-    const int64_t d0 = c.dbase + cv * VEC;
-    const int64_t t0 = c.tt * p.tsteps + lane_t;
+  {
+    const TileCoord& c = s_tc[0];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
-    if (d0 < p.D) {
-      load_f32<VEC>(kd + d0, nk);
-      const int64_t row = c.b * p.L + t0;
-      const T* pd = dh + row * p.D + d0;
-      const T* px = x + row * p.D + d0;
-      const T* pg = gl + row * 2 * p.D + d0;
-#pragma unroll
-      for (int s = 0; s < kTc; ++s) {
-        if (t0 + s < p.L) {
-          ng[s] = IO::load_raw(pd + s * p.D);
-          nx[s] = IO::load_raw(px + s * p.D);
-          nr[s] = IO::load_raw(pg + s * 2 * p.D);
-          ni[s] = IO::load_raw(pg + s * 2 * p.D + p.D);
-        }
-      }
-    }
-  };
-  if (s_tc[0].tile < p.n_tiles_b) fetch(s_tc[0]);
+    if (c.tile < p.n_tiles_b && c.dbase + cv * VEC < p.D) load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
+  }
 
   for (int it = 0;; ++it) {
+    const int stage = it % S;
     const int buf = it & 1;
-    const TileCoord tc = s_tc[it % 3];
+    const TileCoord tc = s_tc[it % RING];
     if (tc.tile >= p.n_tiles_b) break;
     const int64_t d0 = tc.dbase + cv * VEC;
     const bool ch_ok = d0 < p.D;
-    const int64_t t0 = tc.tt * p.tsteps + lane_t;
-    // the ticket after next: drawn now, decoded before the barrier
+    const int64_t t0 = tc.tt * p.tsteps + row0;
+    int64_t left = ch_ok ? p.L - t0 : 0;
+    const int valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
     const uint32_t ticket = drawer ? atomicAdd(&bh->ticket, 1u) : 0u;
-
-    // 1. gates kept as E = expm1(l), r, i (with x and dh); chunk maps of both directions
     float k[VEC];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) k[v] = nk[v];
-    float xv[kTc][VEC], rv[kTc][VEC], iv[kTc][VEC], gv[kTc][VEC], ev[kTc][VEC];
-    float A[VEC], U[VEC], W[VEC];
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      A[v] = 1.0f;
-      U[v] = 0.0f;
-      W[v] = 0.0f;
-    }
-#pragma unroll
-    for (int s = 0; s < kTc; ++s) {
-      const bool ok = ch_ok && t0 + s < p.L;
-      IO::unpack(ng[s], gv[s]);
-      IO::unpack(nx[s], xv[s]);
-      IO::unpack(nr[s], rv[s]);
-      IO::unpack(ni[s], iv[s]);
-#pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        if (ok) {
-          const float r = M::sigmoid(rv[s][v]);
-          const float i = M::sigmoid(iv[s][v]);
-          const float e = M::expm1_nonpos(k[v] * r);
-          const float alpha = 1.0f + e;
-          const float uu = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
-          rv[s][v] = r;
-          iv[s][v] = i;
-          ev[s][v] = e;
-          U[v] = fmaf(alpha, U[v], uu);
-          A[v] *= alpha;                      // prod of alpha up to and including s
-          W[v] = fmaf(A[v], gv[s][v], W[v]);  // w at the chunk start from a zero carry
-        } else {  // the identity: alpha = 1, no input, no upstream gradient
-          rv[s][v] = 0.0f;
-          iv[s][v] = 0.0f;
-          ev[s][v] = 0.0f;
-          gv[s][v] = 0.0f;
-          xv[s][v] = 0.0f;
-        }
-      }
-    }
     {
-      const TileCoord nc = s_tc[(it + 1) % 3];
-      if (nc.tile < p.n_tiles_b) fetch(nc);
+      const TileCoord& c = s_tc[(it + 1) % RING];
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+      if (c.tile < p.n_tiles_b && c.dbase + cv * VEC < p.D)
+        load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
+    }
+
+    // 1. the stage's rows, gates kept as E, r, i; chunk maps of both directions
+    mbar_wait(&bars[stage], (uint32_t)(it / S) & 1u, &fh->err);
+    const unsigned char* sb = smem + (size_t)stage * NB * box_bytes<T>();
+    float gv[kTc][VEC], xv[kTc][VEC], ev[kTc][VEC], rv[kTc][VEC], iv[kTc][VEC];
+    float A[VEC], U[VEC], W[VEC];
+    {
+      Raw rg[kTc], rx[kTc], rr[kTc], ri[kTc];
+      lds_rows<IO>(sb, row0, cv, rg);
+      lds_rows<IO>(sb + box_bytes<T>(), row0, cv, rx);
+      lds_rows<IO>(sb + 2 * box_bytes<T>(), row0, cv, rr);
+      lds_rows<IO>(sb + 3 * box_bytes<T>(), row0, cv, ri);
+      if (valid == kTc)
+        bwd_chunk<IO, M, true>(k, rg, rx, rr, ri, valid, gv, xv, ev, rv, iv, A, U, W);
+      else
+        bwd_chunk<IO, M, false>(k, rg, rx, rr, ri, valid, gv, xv, ev, rv, iv, A, U, W);
     }
     // 2. warp maps: h forwards (prefix), w backwards (suffix)
     float A2[VEC];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) A2[v] = A[v];
-    float ea[VEC], eu[VEC], wa[VEC], wu[VEC], sa[VEC], sw[VEC], wa2[VEC], ww[VEC];
-    warp_prefix<VEC>(A, U, tcl, cv, ea, eu, wa, wu);
-    warp_suffix<VEC>(A2, W, tcl, cv, sa, sw, wa2, ww);
+    float ea[VEC], eu[VEC], sa[VEC], sw[VEC];
+    warp_prefix<VEC>(A, U, tcl, ea, eu);
+    warp_suffix<VEC>(A2, W, tcl, sa, sw);
     if (tcl == kNtl - 1) {
 #pragma unroll
       for (int v = 0; v < VEC; ++v) {
-        s_wa[buf][warp][cv * VEC + v] = wa[v];
-        s_wu[buf][warp][cv * VEC + v] = wu[v];
+        s_wa[buf][warp][cv * VEC + v] = A[v];
+        s_wu[buf][warp][cv * VEC + v] = U[v];
       }
     }
     if (tcl == 0) {
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) s_ww[buf][warp][cv * VEC + v] = ww[v];
+      for (int v = 0; v < VEC; ++v) s_ww[buf][warp][cv * VEC + v] = W[v];
     }
-    if (drawer) s_tc[(it + 2) % 3] = decode(ticket);
-    __syncthreads();
+    if (drawer) s_tc[(it + S + 1) % RING] = decode(ticket);
+    __syncthreads();  // the stage is read: refill it with the tile S ahead
+    if (threadIdx.x == 0) {
+      const TileCoord& c = s_tc[(it + S) % RING];
+      if (c.tile < p.n_tiles_b) issue(stage, c);
+    }
 
     // 3. warp 0, one lane per channel: warp prefix / suffix maps, the h carry
     //    from the forward, the w carry by look-back from the later tiles
@@ -635,9 +806,9 @@ __global__ void __launch_bounds__(kMaxWarps * 32, sizeof(T) == 4 ? 2 : 3)
         wn[v] = (1.0f + ev[s][v]) * g;
       }
     }
-    const int64_t row0 = tc.b * p.L + t0;
-    T* pdx = dx + row0 * p.D + d0;
-    T* pdg = dgl + row0 * 2 * p.D + d0;
+    const int64_t row = tc.b * p.L + t0;
+    T* pdx = dx + row * p.D + d0;
+    T* pdg = dgl + row * 2 * p.D + d0;
 #pragma unroll
     for (int s = 0; s < kTc; ++s) {
       float ox[VEC], orho[VEC], oiota[VEC];
@@ -646,9 +817,8 @@ __global__ void __launch_bounds__(kMaxWarps * 32, sizeof(T) == 4 ? 2 : 3)
         const float e = ev[s][v], r = rv[s][v], i = iv[s][v], g = gv[s][v];
         const float alpha = 1.0f + e;
         const float q = -e * (2.0f + e);
-        const float beta = M::sqrt(q) * i;
-        const float uu = beta * xv[s][v];
-        const float c2 = (q > 0.0f) ? M::div(alpha * uu, q) : 0.0f;  // alpha i x / n
+        float beta, uu, c2;  // beta = n i, u = beta x, c2 = alpha u / q = alpha i x / n
+        M::norm_terms(q, i, xv[s][v], alpha, beta, uu, c2);
         const float dl = g * alpha * (hs[v] - c2);
         orho[v] = dl * k[v] * (r - r * r);
         oiota[v] = g * uu * (1.0f - i);
@@ -656,7 +826,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, sizeof(T) == 4 ? 2 : 3)
         dlr[v] = fmaf(dl, r, dlr[v]);
         hs[v] = fmaf(alpha, hs[v], uu);
       }
-      if (ch_ok && t0 + s < p.L) {
+      if (s < valid) {
         IO::store(pdx + s * p.D, ox);
         IO::store(pdg + s * 2 * p.D, orho);
         IO::store(pdg + s * 2 * p.D + p.D, oiota);
@@ -736,7 +906,7 @@ __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
         const float k = s_k[threadIdx.x * VEC + v];
         const float rr = M::sigmoid(rv[r][v]);
         const float i = M::sigmoid(iv[r][v]);
-        const float e = M::expm1_nonpos(k * rr);
+        const float e = M::expm1_any(k * rr);
         out[v] = fmaf(1.0f + e, hp[r][v], M::sqrt(-e * (2.0f + e)) * i * xv[r][v]);
       }
 #pragma unroll
