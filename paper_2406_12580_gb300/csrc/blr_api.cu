@@ -238,7 +238,7 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
   a.h = h;
   a.h_last = h_last;
   a.ws = w;
-  const int threads = plan.nwarps * 32;
+  const int threads = (plan.nwarps + 1) * 32;  // consumer warps + the scanner warp
   unsigned grid = 1;
   if (desc->io == BLR_F32) {
     auto k = blr::scan_fwd_kernel<float, blr::MathPrecise>;

@@ -251,11 +251,11 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
 __device__ __noinline__ bool wait_record(const uint32_t* pre, const unsigned long long* agg,
                                          uint32_t* err, uint64_t timeout_ns) {
   const uint64_t start = global_timer_ns();
-  uint32_t sleep_ns = 32;
+  uint32_t sleep_ns = 16;
   for (uint32_t iter = 0;; ++iter) {
     if (ld_record(pre) != kEmpty || !agg_empty(ld_record(agg))) return true;
     __nanosleep(sleep_ns);
-    if (sleep_ns < 512) sleep_ns <<= 1;
+    if (sleep_ns < 128) sleep_ns <<= 1;
     if ((iter & 7u) == 7u) {
       if (*reinterpret_cast<volatile uint32_t*>(err) & kErrTimeout) return false;
       if (global_timer_ns() - start > timeout_ns || iter > kMaxWaitIters) {

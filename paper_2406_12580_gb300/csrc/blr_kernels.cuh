@@ -183,42 +183,63 @@ __device__ __forceinline__ void warp_suffix(float (&A)[V], float (&W)[V], int tc
 // trip; the walk folds aggregates (nearest first) until it meets a published
 // prefix. The farthest predecessor (i = nprev - 1, the first tile of the
 // chain) publishes only a prefix, so the walk always ends.
+// The first window's loads, issued early so that their round trip overlaps
+// other work (predecessors past the first tile are not read).
+struct LookWindow {
+  uint32_t pr[kLookWindow];
+  unsigned long long ag[kLookWindow];
+};
+
+__device__ __forceinline__ void lookback_load(const unsigned long long* agg, const uint32_t* pre,
+                                              int64_t step, int64_t nprev, int64_t i,
+                                              LookWindow& w) {
+#pragma unroll
+  for (int q = 0; q < kLookWindow; ++q) {
+    w.pr[q] = kEmpty;
+    w.ag[q] = ~0ull;
+    if (i + q < nprev) {
+      w.pr[q] = ld_record(pre + (i + q) * step);
+      w.ag[q] = ld_record(agg + (i + q) * step);
+    }
+  }
+}
+
+// Walks the predecessors starting with the window `w` (loaded for i = 0).
 __device__ __forceinline__ float lookback(const unsigned long long* agg, const uint32_t* pre,
-                                          int64_t step, int64_t nprev, uint32_t* err) {
+                                          int64_t step, int64_t nprev, uint32_t* err,
+                                          LookWindow& w) {
   float ea = 1.0f, eu = 0.0f;  // fold of the predecessors walked so far
   int64_t i = 0;
   for (;;) {
-    uint32_t pr[kLookWindow];
-    unsigned long long ag[kLookWindow];
-#pragma unroll
-    for (int q = 0; q < kLookWindow; ++q) {
-      pr[q] = kEmpty;
-      ag[q] = ~0ull;
-      if (i + q < nprev) {
-        pr[q] = ld_record(pre + (i + q) * step);
-        ag[q] = ld_record(agg + (i + q) * step);
-      }
-    }
     int adv = kLookWindow;
     bool open = true, wait = false;
 #pragma unroll
     for (int q = 0; q < kLookWindow; ++q) {
       if (open) {
-        if (pr[q] != kEmpty) return fmaf(ea, __uint_as_float(pr[q]), eu);
-        if (agg_empty(ag[q])) {  // published nothing yet: wait for it, then re-read from it
+        if (w.pr[q] != kEmpty) return fmaf(ea, __uint_as_float(w.pr[q]), eu);
+        if (agg_empty(w.ag[q])) {  // published nothing yet: wait for it, then re-read from it
           open = false;
           wait = true;
           adv = q;
         } else {
-          eu = fmaf(ea, __uint_as_float((uint32_t)(ag[q] >> 32)), eu);
-          ea *= __uint_as_float((uint32_t)ag[q]);
+          eu = fmaf(ea, __uint_as_float((uint32_t)(w.ag[q] >> 32)), eu);
+          ea *= __uint_as_float((uint32_t)w.ag[q]);
         }
       }
     }
     if (wait && !wait_record(pre + (i + adv) * step, agg + (i + adv) * step, err, kWaitTimeoutNs))
       return eu;  // the wait expired (recorded): finish with what is known
     i += adv;
+    lookback_load(agg, pre, step, nprev, i, w);
   }
+}
+
+// The whole walk, loads included.
+__device__ __forceinline__ float lookback(const unsigned long long* agg, const uint32_t* pre,
+                                          int64_t step, int64_t nprev, uint32_t* err) {
+  LookWindow w;
+  lookback_load(agg, pre, step, nprev, 0, w);
+  return lookback(agg, pre, step, nprev, err, w);
 }
 
 // ------------------------------------------------------------ tile tickets
@@ -236,17 +257,21 @@ struct TileCoord {
   int64_t dbase;  // first channel of the group
 };
 
+// Tile counts stay below 2^30 (checked on the host), so 32-bit division suffices.
 __device__ __forceinline__ TileCoord decode_tile(int64_t tile, int64_t n_tiles, int64_t n_c,
                                                  int64_t n_cg, int ch, int64_t n_t, bool reverse) {
   TileCoord c;
   c.tile = tile;
   c.tt = c.cidx = c.b = c.dbase = 0;
   if (tile < n_tiles) {
-    const int64_t q = tile / n_c;
-    c.tt = reverse ? n_t - 1 - q : q;  // the backward hands tiles out from the end
-    c.cidx = tile - q * n_c;
-    c.b = c.cidx / n_cg;
-    c.dbase = (c.cidx - c.b * n_cg) * ch;
+    const uint32_t t32 = (uint32_t)tile, nc32 = (uint32_t)n_c, ncg32 = (uint32_t)n_cg;
+    const uint32_t q = t32 / nc32;
+    const uint32_t cidx = t32 - q * nc32;
+    const uint32_t b = cidx / ncg32;
+    c.tt = reverse ? n_t - 1 - (int64_t)q : (int64_t)q;  // the backward hands tiles out from the end
+    c.cidx = cidx;
+    c.b = b;
+    c.dbase = (int64_t)(cidx - b * ncg32) * ch;
   }
   return c;
 }
@@ -327,9 +352,18 @@ __device__ __forceinline__ void fwd_chunk(const float (&k)[4],
 }
 
 // ---------------------------------------------------------------- forward scan
+//
+// Block = nwarps consumer warps (one time sub-tile each) + one scanner warp,
+// one barrier per tile. In iteration k the consumers compute tile k's gates
+// and maps while the scanner finishes tile k-1: it combines the consumers'
+// warp maps, publishes the tile's aggregate, walks back for the carry,
+// publishes the prefix and writes every warp's starting state; it also draws
+// tickets and refills the freed stage. After the barrier the consumers apply
+// tile k-1 (whose alpha and u they kept in registers). The scanner's
+// round trips to L2 thus overlap the consumers' arithmetic.
 
 template <typename T, class M>
-__global__ void __launch_bounds__(kMaxWarps * 32, 4)
+__global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
     scan_fwd_kernel(const __grid_constant__ FwdArgs a) {
   using IO = Io<T, 4>;
   using Raw = typename IO::Raw;
@@ -338,15 +372,17 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 4)
   constexpr int S = fwd_stages<T>();
   constexpr int NB = 3;  // boxes per stage: x, rho, iota
   constexpr int RING = S + 2;
-  static_assert(CH == 32, "warp 0 handles one channel per lane");
+  static_assert(CH == 32, "the scanner handles one channel per lane");
   const Plan& p = a.p;
+  const int nw = p.nwarps;  // consumer warps
 
   extern __shared__ __align__(1024) unsigned char dyn_smem[];
   unsigned char* smem = ring_base(dyn_smem);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * NB * box_bytes<T>());
-  __shared__ float2 s_wmap[2][kMaxWarps][CH];  // warp maps, then warp prefix maps
-  __shared__ float s_carry[2][CH];
+  __shared__ float2 s_wtot[2][kMaxWarps][CH];  // each warp's map of its sub-tile
+  __shared__ float s_hw[2][kMaxWarps][CH];     // each warp's starting state
   __shared__ TileCoord s_tc[RING];
+  __shared__ int s_done[2];                    // consumer warps past their maps
 
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
   unsigned long long* agg = reinterpret_cast<unsigned long long*>(a.ws + p.off_fagg);
@@ -355,11 +391,11 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 4)
   T* h = static_cast<T*>(a.h);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool scanner = warp == nw;
   const int cv = lane % kNvl, tcl = lane / kNvl;
   const int64_t BD = p.B * p.D;
   const int row0 = warp * kWarpSteps + tcl * kTc;  // this lane's first row in a tile
   const uint32_t box_tx = (uint32_t)p.tsteps * CH * sizeof(T);
-  const bool drawer = threadIdx.x == blockDim.x - 1;  // draws the tickets
 
   auto decode = [&](uint32_t t) {
     return decode_tile((int64_t)t, p.n_tiles_f, p.n_c_f, p.n_cg_f, CH, p.n_t, false);
@@ -373,133 +409,184 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 4)
     tma_load_3d(dst + 2 * box_bytes<T>(), &a.tm_gl, &bars[stage], (int)p.D + d, t, bb);
   };
 
+  // Prologue: thread 0 draws the first S tiles and starts their loads.
+  if (threadIdx.x < 2) s_done[threadIdx.x] = 0;
   if (threadIdx.x == 0) {
     for (int j = 0; j < S; ++j) mbar_init(&bars[j], 1);
     fence_mbar_init();
-  }
-  if (drawer) {
-    for (int j = 0; j <= S; ++j) s_tc[j] = decode(atomicAdd(&fh->ticket, 1u));
+    for (int j = 0; j < S; ++j) {
+      s_tc[j] = decode(atomicAdd(&fh->ticket, 1u));
+      if (s_tc[j].tile < p.n_tiles_f) issue(j, s_tc[j]);
+    }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int j = 0; j < S; ++j)
-      if (s_tc[j].tile < p.n_tiles_f) issue(j, s_tc[j]);
-  }
-  float nk[VEC];  // k of the next tile's channels
-  {
-    const TileCoord& c = s_tc[0];
+
+  // Consumer state carried from tile k-1 to its apply in iteration k.
+  float pal[kTc][VEC], pu[kTc][VEC], pea[VEC], peu[VEC];
+  TileCoord prev;
+  prev.tile = p.n_tiles_f;  // none
+  prev.tt = prev.cidx = prev.b = prev.dbase = 0;
+  int prev_valid = 0;
+  float nk[VEC];
 #pragma unroll
-    for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
-    if (c.tile < p.n_tiles_f && c.dbase + cv * VEC < p.D) load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
-  }
+  for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+  if (!scanner && s_tc[0].tile < p.n_tiles_f && s_tc[0].dbase + cv * VEC < p.D)
+    load_f32<VEC>(kd + s_tc[0].dbase + cv * VEC, nk);
 
   for (int it = 0;; ++it) {
-    const int stage = it % S;
-    const int buf = it & 1;
     const TileCoord tc = s_tc[it % RING];
-    if (tc.tile >= p.n_tiles_f) break;
-    const int64_t d0 = tc.dbase + cv * VEC;
-    const bool ch_ok = d0 < p.D;
-    const int64_t t0 = tc.tt * p.tsteps + row0;
-    int64_t left = ch_ok ? p.L - t0 : 0;
-    const int valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
-    const uint32_t ticket = drawer ? atomicAdd(&fh->ticket, 1u) : 0u;  // decoded before B1
-    float k[VEC];
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) k[v] = nk[v];
-    {
-      const TileCoord& c = s_tc[(it + 1) % RING];
-#pragma unroll
-      for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
-      if (c.tile < p.n_tiles_f && c.dbase + cv * VEC < p.D)
-        load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
-    }
+    const bool cur_ok = tc.tile < p.n_tiles_f;
+    const bool prev_ok = prev.tile < p.n_tiles_f;
+    if (!cur_ok && !prev_ok) break;
+    const int buf = it & 1;
 
-    // 1. the stage's rows of this lane, gates, chunk map
-    mbar_wait(&bars[stage], (uint32_t)(it / S) & 1u, &fh->err);
-    const unsigned char* sb = smem + (size_t)stage * NB * box_bytes<T>();
-    Raw rx[kTc], rr[kTc], ri[kTc];
-    lds_rows<IO>(sb, row0, cv, rx);
-    lds_rows<IO>(sb + box_bytes<T>(), row0, cv, rr);
-    lds_rows<IO>(sb + 2 * box_bytes<T>(), row0, cv, ri);
-    float al[kTc][VEC], u[kTc][VEC];
-    if (valid == kTc)
-      fwd_chunk<IO, M, true>(k, rx, rr, ri, valid, al, u);
-    else
-      fwd_chunk<IO, M, false>(k, rx, rr, ri, valid, al, u);
-    float A[VEC], U[VEC];
+    if (!scanner) {
+      // ---- consumers: tile it, gates and maps
+      float al[kTc][VEC], u[kTc][VEC], ea[VEC], eu[VEC];
+      int valid = 0;
+      if (cur_ok) {
+        const int64_t d0 = tc.dbase + cv * VEC;
+        const int64_t left = (d0 < p.D) ? p.L - (tc.tt * p.tsteps + row0) : 0;
+        valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
+        float k[VEC];
 #pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      A[v] = al[0][v];
-      U[v] = u[0][v];
+        for (int v = 0; v < VEC; ++v) k[v] = nk[v];
+        {
+          const TileCoord& c = s_tc[(it + 1) % RING];
 #pragma unroll
-      for (int s = 1; s < kTc; ++s) {
-        U[v] = fmaf(al[s][v], U[v], u[s][v]);
-        A[v] *= al[s][v];
-      }
-    }
-    // 2. warp prefix maps
-    float ea[VEC], eu[VEC];
-    warp_prefix<VEC>(A, U, tcl, ea, eu);
-    if (tcl == kNtl - 1) {
-#pragma unroll
-      for (int v = 0; v < VEC; ++v) s_wmap[buf][warp][cv * VEC + v] = make_float2(A[v], U[v]);
-    }
-    if (drawer) s_tc[(it + S + 1) % RING] = decode(ticket);
-    __syncthreads();  // the stage is read: refill it with the tile S ahead
-    if (threadIdx.x == 0) {
-      const TileCoord& c = s_tc[(it + S) % RING];
-      if (c.tile < p.n_tiles_f) issue(stage, c);
-    }
-
-    // 3. warp 0, one lane per channel: tile map, look-back, tile prefix
-    if (warp == 0) {
-      const int ch = lane;
-      const bool cval = tc.dbase + ch < p.D;
-      float pa = 1.0f, pu = 0.0f;
-      for (int w = 0; w < p.nwarps; ++w) {
-        const float2 e = s_wmap[buf][w][ch];
-        s_wmap[buf][w][ch] = make_float2(pa, pu);
-        pu = fmaf(e.x, pu, e.y);
-        pa *= e.x;
-      }
-      float carry = 0.0f;
-      if (cval) {
-        const int64_t rec = tc.tt * BD + tc.b * p.D + tc.dbase + ch;
-        if (tc.tt == 0) {
-          if (a.h0 != nullptr) carry = a.h0[tc.b * p.D + tc.dbase + ch];
-        } else {
-          st_record(&agg[rec], pack_agg(pa, pu));
-          carry = lookback(agg + rec - BD, pre + rec - BD, -BD, tc.tt, &fh->err);
+          for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
+          if (c.tile < p.n_tiles_f && c.dbase + cv * VEC < p.D)
+            load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
         }
-        const float incl = fmaf(pa, carry, pu);
-        st_record(&pre[rec], __float_as_uint(incl));
-        if (tc.tt == p.n_t - 1 && a.h_last != nullptr) a.h_last[tc.b * p.D + tc.dbase + ch] = incl;
-      }
-      s_carry[buf][ch] = carry;
-    }
-    __syncthreads();
-
-    // 4. re-run the chunk from its true starting state
-    if (h != nullptr && ch_ok) {
-      float hs[VEC];
-#pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        const float2 wm = s_wmap[buf][warp][cv * VEC + v];
-        hs[v] = fmaf(ea[v], fmaf(wm.x, s_carry[buf][cv * VEC + v], wm.y), eu[v]);
-      }
-      T* ph = h + (tc.b * p.L + t0) * p.D + d0;
-#pragma unroll
-      for (int s = 0; s < kTc; ++s) {
-        float out[VEC];
+        const int stage = it % S;
+        mbar_wait(&bars[stage], (uint32_t)(it / S) & 1u, &fh->err);
+        const unsigned char* sb = smem + (size_t)stage * NB * box_bytes<T>();
+        Raw rx[kTc], rr[kTc], ri[kTc];
+        lds_rows<IO>(sb, row0, cv, rx);
+        lds_rows<IO>(sb + box_bytes<T>(), row0, cv, rr);
+        lds_rows<IO>(sb + 2 * box_bytes<T>(), row0, cv, ri);
+        if (valid == kTc)
+          fwd_chunk<IO, M, true>(k, rx, rr, ri, valid, al, u);
+        else
+          fwd_chunk<IO, M, false>(k, rx, rr, ri, valid, al, u);
+        float A[VEC], U[VEC];
 #pragma unroll
         for (int v = 0; v < VEC; ++v) {
-          hs[v] = fmaf(al[s][v], hs[v], u[s][v]);
-          out[v] = hs[v];
+          A[v] = al[0][v];
+          U[v] = u[0][v];
+#pragma unroll
+          for (int s = 1; s < kTc; ++s) {
+            U[v] = fmaf(al[s][v], U[v], u[s][v]);
+            A[v] *= al[s][v];
+          }
         }
-        if (s < valid) IO::store(ph + s * p.D, out);
+        warp_prefix<VEC>(A, U, tcl, ea, eu);
+        if (tcl == kNtl - 1) {
+#pragma unroll
+          for (int v = 0; v < VEC; ++v) s_wtot[buf][warp][cv * VEC + v] = make_float2(A[v], U[v]);
+        }
+        // The last consumer warp to get here publishes the tile's aggregate at
+        // once: successors in time may be waiting for it.
+        __syncwarp();
+        __threadfence_block();
+        int last = 0;
+        if (lane == 0) last = atomicAdd(&s_done[buf], 1) == nw - 1;
+        last = __shfl_sync(kFull, last, 0);
+        if (last) {
+          __threadfence_block();
+          const int ch = lane;
+          if (tc.tt > 0 && tc.dbase + ch < p.D) {
+            float pa = 1.0f, pu2 = 0.0f;
+            for (int w = 0; w < nw; ++w) {
+              const float2 e = s_wtot[buf][w][ch];
+              pu2 = fmaf(e.x, pu2, e.y);
+              pa *= e.x;
+            }
+            st_record(&agg[tc.tt * BD + tc.b * p.D + tc.dbase + ch], pack_agg(pa, pu2));
+          }
+          if (lane == 0) s_done[buf] = 0;
+        }
       }
+      __syncthreads();
+      // ---- consumers: apply tile it-1 from the starting states the scanner wrote
+      if (prev_ok && h != nullptr && prev_valid > 0) {
+        const int64_t d0 = prev.dbase + cv * VEC;
+        const int64_t t0 = prev.tt * p.tsteps + row0;
+        float hs[VEC];
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) hs[v] = fmaf(pea[v], s_hw[buf ^ 1][warp][cv * VEC + v], peu[v]);
+        T* ph = h + (prev.b * p.L + t0) * p.D + d0;
+#pragma unroll
+        for (int s = 0; s < kTc; ++s) {
+          float out[VEC];
+#pragma unroll
+          for (int v = 0; v < VEC; ++v) {
+            hs[v] = fmaf(pal[s][v], hs[v], pu[s][v]);
+            out[v] = hs[v];
+          }
+          if (s < prev_valid) IO::store(ph + s * p.D, out);
+        }
+      }
+#pragma unroll
+      for (int s = 0; s < kTc; ++s)
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) {
+          pal[s][v] = al[s][v];
+          pu[s][v] = u[s][v];
+        }
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        pea[v] = ea[v];
+        peu[v] = eu[v];
+      }
+      prev_valid = valid;
+    } else {
+      // ---- scanner: tile it-1's carry and warp states, the next ticket and
+      // the freed stage's refill. The first look-back window and the ticket
+      // are requested before anything else, so their round trips overlap.
+      const int ch = lane;
+      const bool cval = prev_ok && prev.dbase + ch < p.D;
+      const int64_t rec = prev.tt * BD + prev.b * p.D + prev.dbase + ch;
+      LookWindow win;
+      if (cval && prev.tt > 0) lookback_load(agg + rec - BD, pre + rec - BD, -BD, prev.tt, 0, win);
+      uint32_t ticket = 0;
+      if (lane == 0) {
+        ticket = atomicAdd(&fh->ticket, 1u);  // the tile S ahead
+        if (it > 0) {  // the stage tile it-1 used is free: load tile it-1+S into it
+          const TileCoord& c = s_tc[(it - 1 + S) % RING];
+          if (c.tile < p.n_tiles_f) issue((it - 1) % S, c);
+        }
+      }
+      if (prev_ok) {
+        float pa = 1.0f, pu2 = 0.0f;  // the tile's map
+        for (int w = 0; w < nw; ++w) {
+          const float2 e = s_wtot[buf ^ 1][w][ch];
+          pu2 = fmaf(e.x, pu2, e.y);
+          pa *= e.x;
+        }
+        float carry = 0.0f;
+        if (cval) {
+          if (prev.tt == 0) {
+            if (a.h0 != nullptr) carry = a.h0[prev.b * p.D + prev.dbase + ch];
+          } else {
+            carry = lookback(agg + rec - BD, pre + rec - BD, -BD, prev.tt, &fh->err, win);
+          }
+          const float incl = fmaf(pa, carry, pu2);
+          st_record(&pre[rec], __float_as_uint(incl));
+          if (prev.tt == p.n_t - 1 && a.h_last != nullptr)
+            a.h_last[prev.b * p.D + prev.dbase + ch] = incl;
+        }
+        float hw = carry;  // each warp's starting state: the carry through the warps before it
+        for (int w = 0; w < nw; ++w) {
+          s_hw[buf ^ 1][w][ch] = hw;
+          const float2 e = s_wtot[buf ^ 1][w][ch];
+          hw = fmaf(e.x, hw, e.y);
+        }
+      }
+      if (lane == 0) s_tc[(it + S) % RING] = decode(ticket);
+      __syncthreads();
     }
+    prev = tc;
   }
   // The last block out marks the forward complete (for the backward's check).
   __syncthreads();
