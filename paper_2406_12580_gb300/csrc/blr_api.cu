@@ -12,7 +12,7 @@
 #include <cudaTypedefs.h>
 
 #include "blr.h"
-#include "blr_kernels.cuh"
+#include "blr_chain.cuh"
 
 namespace {
 
@@ -48,7 +48,7 @@ blr_status check_desc(const blr_desc* d, Plan* plan, bool* empty_bd) {
   if (d->D % 8 != 0) return fail(BLR_ERR_UNSUPPORTED, "D=%lld is not a multiple of 8", (long long)d->D);
   *empty_bd = (d->B == 0 || d->D == 0);
   if (*empty_bd || d->L == 0) return BLR_OK;
-  // Element offsets (b L + t) 2D + d must fit in int64; tile tickets in int32.
+  // Element offsets (b L + t) 2D + d must fit in int64; tile numbers in int32.
   if (d->B > (int64_t)1 << 40 || d->L > (int64_t)1 << 40 || d->D > (int64_t)1 << 24 ||
       (double)d->B * (double)d->L * (double)d->D > 1e18)
     return fail(BLR_ERR_UNSUPPORTED, "problem too large");
@@ -172,6 +172,53 @@ blr_status make_tensor_map(CUtensorMap* map, const void* base, int io, int64_t c
   return BLR_OK;
 }
 
+// Launches a scan kernel cooperatively: its blocks wait on one another, so
+// all of them must be resident at once.
+template <typename K, typename A>
+blr_status launch_cooperative(K kernel, unsigned grid, int threads, size_t smem, cudaStream_t st,
+                              const A& args, const char* what) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3((unsigned)threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cuda_check(cudaLaunchKernelEx(&cfg, kernel, args), what);
+}
+
+// Grid of a warp-chain kernel: one warp per (batch row, channel group),
+// four warps per block.
+unsigned chain_grid(const Plan& p) {
+  const int64_t warps = p.B * ((p.D + 4 * p.nvl - 1) / (4 * p.nvl));
+  return (unsigned)((warps + 3) / 4);
+}
+
+template <typename T, class M>
+blr_status launch_chain_fwd(const blr::ChainFwdArgs& a, cudaStream_t st) {
+  const unsigned grid = chain_grid(a.p);
+  switch (a.p.nvl) {
+    case 8: blr::chain_fwd_kernel<T, M, 8><<<grid, 128, 0, st>>>(a); break;
+    case 4: blr::chain_fwd_kernel<T, M, 4><<<grid, 128, 0, st>>>(a); break;
+    default: blr::chain_fwd_kernel<T, M, 2><<<grid, 128, 0, st>>>(a); break;
+  }
+  return cuda_check(cudaGetLastError(), "launch chain_fwd_kernel");
+}
+
+template <typename T, class M>
+blr_status launch_chain_bwd(const blr::ChainBwdArgs& a, cudaStream_t st) {
+  const unsigned grid = chain_grid(a.p);
+  switch (a.p.nvl) {
+    case 8: blr::chain_bwd_kernel<T, M, 8><<<grid, 128, 0, st>>>(a); break;
+    case 4: blr::chain_bwd_kernel<T, M, 4><<<grid, 128, 0, st>>>(a); break;
+    default: blr::chain_bwd_kernel<T, M, 2><<<grid, 128, 0, st>>>(a); break;
+  }
+  return cuda_check(cudaGetLastError(), "launch chain_bwd_kernel");
+}
+
 // Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
 // empty record pattern and writes k = -c softplus(Lambda).
 blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fill,
@@ -225,10 +272,17 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
-  // Clear the forward header (tickets, counters, error word), empty the
+  if (plan.chain) {  // warp chains: no look-back records to empty
+    BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), nullptr, 0,
+                        reinterpret_cast<float*>(w + plan.off_k), lambda, desc->D, desc->c, st));
+    const blr::ChainFwdArgs ca{plan, x, gate_logits, h0, h, h_last, w};
+    if (desc->io == BLR_F32) return launch_chain_fwd<float, blr::MathPrecise>(ca, st);
+    return launch_chain_fwd<__nv_bfloat16, blr::MathFast>(ca, st);
+  }
+  // Clear the forward header (counters, error word), empty the
   // forward records, precompute k = -c softplus(Lambda).
-  BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fagg,
-                      plan.off_bagg - plan.off_fagg, reinterpret_cast<float*>(w + plan.off_k),
+  BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fpre,
+                      plan.off_bagg - plan.off_fpre, reinterpret_cast<float*>(w + plan.off_k),
                       lambda, desc->D, desc->c, st));
   blr::FwdArgs a;
   BLR_TRY(make_tensor_map(&a.tm_x, x, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
@@ -244,14 +298,14 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
     auto k = blr::scan_fwd_kernel<float, blr::MathPrecise>;
     const size_t smem = blr::ring_bytes<float, blr::fwd_stages<float>(), 3>();
     BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
-    k<<<grid, threads, smem, st>>>(a);
+    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel"));
   } else {
     auto k = blr::scan_fwd_kernel<__nv_bfloat16, blr::MathFast>;
     const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::fwd_stages<__nv_bfloat16>(), 3>();
     BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
-    k<<<grid, threads, smem, st>>>(a);
+    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel"));
   }
-  return cuda_check(cudaGetLastError(), "launch scan_fwd_kernel");
+  return BLR_OK;
 }
 
 blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
@@ -286,6 +340,14 @@ blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_la
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
+  if (plan.chain) {  // warp chains: clear the counters and partial sums only
+    BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, nullptr, 0,
+                        reinterpret_cast<float*>(w + plan.off_k), lambda, desc->D, desc->c, st));
+    const blr::ChainBwdArgs ca{plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
+                               dlambda, dh0, w};
+    if (desc->io == BLR_F32) return launch_chain_bwd<float, blr::MathPrecise>(ca, st);
+    return launch_chain_bwd<__nv_bfloat16, blr::MathFast>(ca, st);
+  }
   // Clear the backward header and the dLambda partial sums, empty the backward
   // records (the forward's records stay: they hold the carries).
   BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, w + plan.off_bagg,
@@ -310,14 +372,14 @@ blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_la
     auto k = blr::scan_bwd_kernel<float, blr::MathPrecise>;
     const size_t smem = blr::ring_bytes<float, blr::bwd_stages<float>(), 4>();
     BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
-    k<<<grid, threads, smem, st>>>(a);
+    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel"));
   } else {
     auto k = blr::scan_bwd_kernel<__nv_bfloat16, blr::MathFast>;
     const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::bwd_stages<__nv_bfloat16>(), 4>();
     BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
-    k<<<grid, threads, smem, st>>>(a);
+    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel"));
   }
-  return cuda_check(cudaGetLastError(), "launch scan_bwd_kernel");
+  return BLR_OK;
 }
 
 blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_prev,

@@ -3,9 +3,10 @@
 // elementwise and memory-bound: no tensor cores; 16-byte (or 8-byte) accesses
 // along the channels, the gate arithmetic fused into the loads, float32 state.
 //
-// Scan structure. Persistent thread blocks take tiles (tsteps time steps x CH
-// channels of one batch row) from an atomic ticket counter, time-major, so a
-// tile only ever waits for tiles handed out before it. For one tile:
+// Scan structure. Persistent thread blocks (a cooperative launch: all resident)
+// process tiles (tsteps time steps x CH channels of one batch row) on a static
+// schedule, time-major, so a tile only ever waits for tiles of smaller number,
+// which earlier or concurrent iterations of other blocks process. For one tile:
 //   1. every lane loads its kTc steps x VEC channels, computes the gates and
 //      folds its chunk into one affine map h -> A h + U, serially in registers;
 //   2. the kNtl lanes of a warp that share channels combine their maps with
@@ -98,7 +99,7 @@ struct StepArgs {
 
 // ------------------------------------------------------------ preparation
 //
-// Clears the counters of a scan (tickets, exits, partial sums), fills its
+// Clears the counters of a scan (exits, partial sums), fills its
 // look-back records with the empty pattern, and writes k[d] = -c softplus(Lambda_d).
 
 __global__ void prep_kernel(uint32_t* zero, int64_t zero_words, uint4* fill, int64_t fill_vec4,
@@ -242,15 +243,15 @@ __device__ __forceinline__ float lookback(const unsigned long long* agg, const u
   return lookback(agg, pre, step, nprev, err, w);
 }
 
-// ------------------------------------------------------------ tile tickets
+// ------------------------------------------------------------ tile schedule
 //
-// A ticket is decoded once, by the thread that draws it, into the tile's
-// position. Blocks keep decoded tiles in a ring: the tile being finished, the
-// tiles whose inputs are in flight in the shared-memory stages, and the next
-// one drawn.
+// Static schedule: block c processes tiles c, c + G, c + 2G, ... (G blocks,
+// all resident: the scans are cooperative launches), in order. Tiles are
+// numbered time-major, so a tile only waits for tiles of smaller number, and
+// processing order across blocks follows tile order without any queueing.
 
 struct TileCoord {
-  int64_t tile;   // the ticket; >= the tile count means no tile
+  int64_t tile;   // the tile's number; >= the tile count means no tile
   int64_t tt;     // time tile
   int64_t cidx;   // channel group in [0, B * groups per row)
   int64_t b;      // batch row
@@ -355,12 +356,12 @@ __device__ __forceinline__ void fwd_chunk(const float (&k)[4],
 //
 // Block = nwarps consumer warps (one time sub-tile each) + one scanner warp,
 // one barrier per tile. In iteration k the consumers compute tile k's gates
-// and maps while the scanner finishes tile k-1: it combines the consumers'
-// warp maps, publishes the tile's aggregate, walks back for the carry,
-// publishes the prefix and writes every warp's starting state; it also draws
-// tickets and refills the freed stage. After the barrier the consumers apply
-// tile k-1 (whose alpha and u they kept in registers). The scanner's
-// round trips to L2 thus overlap the consumers' arithmetic.
+// and maps (the last consumer warp to finish publishes the tile's aggregate)
+// while the scanner finishes tile k-1: it walks back for the carry, publishes
+// the prefix, writes every warp's starting state and refills the freed TMA
+// stage. After the barrier the consumers apply tile k-1 (whose alpha and u
+// they kept in registers). The scanner's round trips to L2 thus overlap the
+// consumers' arithmetic.
 
 template <typename T, class M>
 __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
@@ -371,7 +372,6 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
   constexpr int CH = kNvl * VEC;
   constexpr int S = fwd_stages<T>();
   constexpr int NB = 3;  // boxes per stage: x, rho, iota
-  constexpr int RING = S + 2;
   static_assert(CH == 32, "the scanner handles one channel per lane");
   const Plan& p = a.p;
   const int nw = p.nwarps;  // consumer warps
@@ -381,7 +381,6 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * NB * box_bytes<T>());
   __shared__ float2 s_wtot[2][kMaxWarps][CH];  // each warp's map of its sub-tile
   __shared__ float s_hw[2][kMaxWarps][CH];     // each warp's starting state
-  __shared__ TileCoord s_tc[RING];
   __shared__ int s_done[2];                    // consumer warps past their maps
 
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
@@ -397,8 +396,8 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
   const int row0 = warp * kWarpSteps + tcl * kTc;  // this lane's first row in a tile
   const uint32_t box_tx = (uint32_t)p.tsteps * CH * sizeof(T);
 
-  auto decode = [&](uint32_t t) {
-    return decode_tile((int64_t)t, p.n_tiles_f, p.n_c_f, p.n_cg_f, CH, p.n_t, false);
+  auto tile_at = [&](int64_t i) {  // this block's i-th tile
+    return decode_tile(i * gridDim.x + blockIdx.x, p.n_tiles_f, p.n_c_f, p.n_cg_f, CH, p.n_t, false);
   };
   auto issue = [&](int stage, const TileCoord& c) {  // one thread: the tile's boxes into a stage
     unsigned char* dst = smem + (size_t)stage * NB * box_bytes<T>();
@@ -409,14 +408,14 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
     tma_load_3d(dst + 2 * box_bytes<T>(), &a.tm_gl, &bars[stage], (int)p.D + d, t, bb);
   };
 
-  // Prologue: thread 0 draws the first S tiles and starts their loads.
+  // Prologue: thread 0 starts the loads of the block's first S tiles.
   if (threadIdx.x < 2) s_done[threadIdx.x] = 0;
   if (threadIdx.x == 0) {
     for (int j = 0; j < S; ++j) mbar_init(&bars[j], 1);
     fence_mbar_init();
     for (int j = 0; j < S; ++j) {
-      s_tc[j] = decode(atomicAdd(&fh->ticket, 1u));
-      if (s_tc[j].tile < p.n_tiles_f) issue(j, s_tc[j]);
+      const TileCoord c = tile_at(j);
+      if (c.tile < p.n_tiles_f) issue(j, c);
     }
   }
   __syncthreads();
@@ -430,11 +429,14 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
   float nk[VEC];
 #pragma unroll
   for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
-  if (!scanner && s_tc[0].tile < p.n_tiles_f && s_tc[0].dbase + cv * VEC < p.D)
-    load_f32<VEC>(kd + s_tc[0].dbase + cv * VEC, nk);
+  {
+    const TileCoord c0 = tile_at(0);
+    if (!scanner && c0.tile < p.n_tiles_f && c0.dbase + cv * VEC < p.D)
+      load_f32<VEC>(kd + c0.dbase + cv * VEC, nk);
+  }
 
   for (int it = 0;; ++it) {
-    const TileCoord tc = s_tc[it % RING];
+    const TileCoord tc = tile_at(it);
     const bool cur_ok = tc.tile < p.n_tiles_f;
     const bool prev_ok = prev.tile < p.n_tiles_f;
     if (!cur_ok && !prev_ok) break;
@@ -452,7 +454,7 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
 #pragma unroll
         for (int v = 0; v < VEC; ++v) k[v] = nk[v];
         {
-          const TileCoord& c = s_tc[(it + 1) % RING];
+          const TileCoord c = tile_at(it + 1);
 #pragma unroll
           for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
           if (c.tile < p.n_tiles_f && c.dbase + cv * VEC < p.D)
@@ -541,21 +543,17 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
       }
       prev_valid = valid;
     } else {
-      // ---- scanner: tile it-1's carry and warp states, the next ticket and
-      // the freed stage's refill. The first look-back window and the ticket
-      // are requested before anything else, so their round trips overlap.
+      // ---- scanner: tile it-1's carry and warp states, and the freed stage's
+      // refill. The first look-back window is requested before anything else,
+      // so its round trip overlaps the rest.
       const int ch = lane;
       const bool cval = prev_ok && prev.dbase + ch < p.D;
       const int64_t rec = prev.tt * BD + prev.b * p.D + prev.dbase + ch;
       LookWindow win;
       if (cval && prev.tt > 0) lookback_load(agg + rec - BD, pre + rec - BD, -BD, prev.tt, 0, win);
-      uint32_t ticket = 0;
-      if (lane == 0) {
-        ticket = atomicAdd(&fh->ticket, 1u);  // the tile S ahead
-        if (it > 0) {  // the stage tile it-1 used is free: load tile it-1+S into it
-          const TileCoord& c = s_tc[(it - 1 + S) % RING];
-          if (c.tile < p.n_tiles_f) issue((it - 1) % S, c);
-        }
+      if (lane == 0 && it > 0) {  // the stage tile it-1 used is free: load tile it-1+S into it
+        const TileCoord c = tile_at(it - 1 + S);
+        if (c.tile < p.n_tiles_f) issue((it - 1) % S, c);
       }
       if (prev_ok) {
         float pa = 1.0f, pu2 = 0.0f;  // the tile's map
@@ -583,7 +581,6 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
           hw = fmaf(e.x, hw, e.y);
         }
       }
-      if (lane == 0) s_tc[(it + S) % RING] = decode(ticket);
       __syncthreads();
     }
     prev = tc;
@@ -699,7 +696,6 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
   constexpr int CH = kNvl * VEC;
   constexpr int S = bwd_stages<T>();
   constexpr int NB = 4;  // boxes per stage: dh, x, rho, iota
-  constexpr int RING = S + 2;
   static_assert(CH == 32, "warp 0 handles one channel per lane");
   const Plan& p = a.p;
 
@@ -711,7 +707,6 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
   __shared__ float s_ww[2][kMaxWarps][CH];   // warp W          -> warp suffix map W
   __shared__ float s_ws[2][kMaxWarps][CH];   //                 -> warp suffix map A
   __shared__ float s_hc[2][CH], s_wc[2][CH];
-  __shared__ TileCoord s_tc[RING];
   __shared__ int s_flag;
 
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
@@ -729,10 +724,8 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
   const int64_t BD = p.B * p.D;
   const int row0 = warp * kWarpSteps + tcl * kTc;
   const uint32_t box_tx = (uint32_t)p.tsteps * CH * sizeof(T);
-  const bool drawer = threadIdx.x == blockDim.x - 1;
-
-  auto decode = [&](uint32_t t) {
-    return decode_tile((int64_t)t, p.n_tiles_b, p.n_c_b, p.n_cg_b, CH, p.n_t, true);
+  auto tile_at = [&](int64_t i) {  // this block's i-th tile (from the end in time)
+    return decode_tile(i * gridDim.x + blockIdx.x, p.n_tiles_b, p.n_c_b, p.n_cg_b, CH, p.n_t, true);
   };
   auto issue = [&](int stage, const TileCoord& c) {
     unsigned char* dst = smem + (size_t)stage * NB * box_bytes<T>();
@@ -748,22 +741,22 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
     for (int j = 0; j < S; ++j) mbar_init(&bars[j], 1);
     fence_mbar_init();
   }
-  if (drawer) {
+  if (threadIdx.x == 0) {
     const bool ok = __ldcg(&fh->tag) == p.tag && __ldcg(&fh->complete) == 1u;
     if (!ok) atomicOr(&fh->err, kErrWorkspace);
     s_flag = ok;
-    if (ok)
-      for (int j = 0; j <= S; ++j) s_tc[j] = decode(atomicAdd(&bh->ticket, 1u));
   }
   __syncthreads();
   if (!s_flag) return;  // no forward carries for this problem: write nothing
   if (threadIdx.x == 0) {
-    for (int j = 0; j < S; ++j)
-      if (s_tc[j].tile < p.n_tiles_b) issue(j, s_tc[j]);
+    for (int j = 0; j < S; ++j) {
+      const TileCoord c = tile_at(j);
+      if (c.tile < p.n_tiles_b) issue(j, c);
+    }
   }
   float nk[VEC];
   {
-    const TileCoord& c = s_tc[0];
+    const TileCoord c = tile_at(0);
 #pragma unroll
     for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
     if (c.tile < p.n_tiles_b && c.dbase + cv * VEC < p.D) load_f32<VEC>(kd + c.dbase + cv * VEC, nk);
@@ -772,19 +765,18 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
   for (int it = 0;; ++it) {
     const int stage = it % S;
     const int buf = it & 1;
-    const TileCoord tc = s_tc[it % RING];
+    const TileCoord tc = tile_at(it);
     if (tc.tile >= p.n_tiles_b) break;
     const int64_t d0 = tc.dbase + cv * VEC;
     const bool ch_ok = d0 < p.D;
     const int64_t t0 = tc.tt * p.tsteps + row0;
     int64_t left = ch_ok ? p.L - t0 : 0;
     const int valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
-    const uint32_t ticket = drawer ? atomicAdd(&bh->ticket, 1u) : 0u;
     float k[VEC];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) k[v] = nk[v];
     {
-      const TileCoord& c = s_tc[(it + 1) % RING];
+      const TileCoord c = tile_at(it + 1);
 #pragma unroll
       for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
       if (c.tile < p.n_tiles_b && c.dbase + cv * VEC < p.D)
@@ -825,10 +817,9 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
 #pragma unroll
       for (int v = 0; v < VEC; ++v) s_ww[buf][warp][cv * VEC + v] = W[v];
     }
-    if (drawer) s_tc[(it + S + 1) % RING] = decode(ticket);
     __syncthreads();  // the stage is read: refill it with the tile S ahead
     if (threadIdx.x == 0) {
-      const TileCoord& c = s_tc[(it + S) % RING];
+      const TileCoord c = tile_at(it + S);
       if (c.tile < p.n_tiles_b) issue(stage, c);
     }
 

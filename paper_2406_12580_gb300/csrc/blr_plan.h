@@ -2,7 +2,7 @@
 //
 // The (B, L, D) problem is cut into tiles of `tsteps` consecutive time steps x
 // `CH` consecutive channels of one batch row. A thread block scans one tile at
-// a time (persistent blocks take tiles from an atomic ticket counter):
+// a time (persistent blocks, static schedule):
 //   lane (cv, tcl) of warp w owns channels [cv*VEC, cv*VEC + VEC) of the tile
 //   and the kTc steps starting at w*kWarpSteps + tcl*kTc.
 // Tiles of the same (batch row, channel group) are chained along time with a
@@ -40,7 +40,7 @@ constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
 constexpr uint32_t kMaxWaitIters = 1u << 23;
 
 struct FwdHeader {     // cleared before every forward (by its prep kernel)
-  uint32_t ticket;     // tiles handed out
+  uint32_t spare;
   uint32_t exited;     // blocks that left the tile loop
   uint32_t err;        // error bits (forward and backward timeouts, workspace misuse)
   uint32_t tag;        // hash of the problem, written when the forward completed
@@ -49,7 +49,7 @@ struct FwdHeader {     // cleared before every forward (by its prep kernel)
 };
 
 struct BwdHeader {     // cleared before every backward
-  uint32_t ticket;
+  uint32_t spare;
   uint32_t exited;
   uint32_t selftest_flag;  // a flag nothing sets (blr_selftest_wait_timeout)
   uint32_t pad[5];
@@ -60,10 +60,21 @@ struct BwdHeader {     // cleared before every backward
 inline int fwd_vec(int) { return 4; }
 inline int bwd_vec(int) { return 4; }
 
+// Problems with at least this many (batch row, channel group) chains, each at
+// most kChainMaxBlocks blocks long, use the warp-chain kernels (one warp walks
+// one chain); the others the tiled look-back kernels. The choice depends only
+// on the problem's shape.
+constexpr int64_t kChainMinWarps = 2048;
+constexpr int64_t kChainMaxBlocks = 16;
+
 struct Plan {
   int64_t B, L, D;
   int io;           // 0 = float32, 1 = bfloat16
   float c;
+  int chain;        // 1: warp-chain kernels, 0: tiled look-back kernels
+  int nvl;          // warp-chain: lanes along channels (chain width 4 * nvl channels)
+  int64_t bs;       // warp-chain: time steps per block = (32 / nvl) * kTc
+  int64_t n_blk;    // warp-chain: blocks per sequence
   int nwarps;       // warps per block = time sub-tiles per tile
   int64_t tsteps;   // time steps per tile = nwarps * kWarpSteps
   int64_t n_t;      // time tiles
@@ -120,7 +131,24 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   __builtin_memcpy(&cbits, &c, 4);
   h = fnv1a(h, cbits);
   p->tag = h | 1u;  // never 0, the value of a cleared header
-  const size_t rec = (size_t)p->n_t * (size_t)B * (size_t)D;  // one per (time tile, channel)
+  p->chain = 0;
+  p->nvl = 8;
+  for (int nvl = 8; nvl >= 2; nvl >>= 1) {
+    const int64_t warps = B * ((D + 4 * nvl - 1) / (4 * nvl));
+    const int64_t bs = (int64_t)(32 / nvl) * kTc;
+    if (warps >= kChainMinWarps && (L + bs - 1) / bs <= kChainMaxBlocks) {
+      p->chain = 1;
+      p->nvl = nvl;
+      break;
+    }
+  }
+  p->bs = (int64_t)(32 / p->nvl) * kTc;
+  p->n_blk = (L + p->bs - 1) / p->bs;
+  // The forward's states after each time tile (or after each chain block but
+  // the last) are kept for the backward; the tiled kernels also need aggregates
+  // and backward records.
+  const size_t rec = (size_t)(p->chain ? p->n_blk - 1 : p->n_t) * (size_t)B * (size_t)D;
+  const size_t rec_t = p->chain ? 0 : rec;
   size_t o = 0;
   p->off_fhdr = o;
   o = align_up(o + sizeof(FwdHeader), kAlign);
@@ -130,14 +158,14 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   o = align_up(o + 8 * (size_t)kStripes * (size_t)D, kAlign);
   p->off_k = o;
   o = align_up(o + 4 * (size_t)D, kAlign);
-  p->off_fagg = o;  // forward records: agg then pre, filled together
-  o = align_up(o + 8 * rec, kAlign);
-  p->off_fpre = o;
+  p->off_fpre = o;  // forward records: pre then agg, emptied together
   o = align_up(o + 4 * rec, kAlign);
+  p->off_fagg = o;
+  o = align_up(o + 8 * rec_t, kAlign);
   p->off_bagg = o;  // backward records
-  o = align_up(o + 8 * rec, kAlign);
+  o = align_up(o + 8 * rec_t, kAlign);
   p->off_bpre = o;
-  o = align_up(o + 4 * rec, kAlign);
+  o = align_up(o + 4 * rec_t, kAlign);
   p->bytes = o;
 }
 
