@@ -12,7 +12,7 @@
 #include <cudaTypedefs.h>
 
 #include "blr.h"
-#include "blr_chain.cuh"
+#include "blr_seq.cuh"
 
 namespace {
 
@@ -59,6 +59,8 @@ blr_status check_desc(const blr_desc* d, Plan* plan, bool* empty_bd) {
   blr::make_plan(d->B, d->L, d->D, (int)d->io, d->c, plan);
   if (plan->n_tiles_f >= ((int64_t)1 << 30) || plan->n_tiles_b >= ((int64_t)1 << 30))
     return fail(BLR_ERR_UNSUPPORTED, "too many tiles (%lld)", (long long)plan->n_tiles_b);
+  if (plan->seq && plan->n_chain >= ((int64_t)1 << 31))
+    return fail(BLR_ERR_UNSUPPORTED, "too many chains (%lld)", (long long)plan->n_chain);
   return BLR_OK;
 }
 
@@ -152,17 +154,19 @@ blr_status tensor_map_encoder(PFN_cuTensorMapEncodeTiled_v12000* out) {
   return BLR_OK;
 }
 
-// A 3-D tensor map over a row-major (B, L, cols) tensor seen as (cols, L, B),
-// boxes of 32 columns x `rows` steps x 1 batch row; out-of-range elements of
-// a box read as zero.
+// A 3-D tensor map over `cols` columns of a row-major (B, L, row_elems)
+// tensor (row_elems = cols unless given), seen as (cols, L, B); boxes of
+// `box_cols` columns x `rows` steps x 1 batch row. Loads read elements
+// outside the view as zero; stores skip them.
 blr_status make_tensor_map(CUtensorMap* map, const void* base, int io, int64_t cols, int64_t L,
-                           int64_t B, int64_t rows) {
+                           int64_t B, int64_t rows, uint32_t box_cols = 32, int64_t row_elems = 0) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = nullptr;
   BLR_TRY(tensor_map_encoder(&enc));
   const cuuint64_t es = (io == BLR_F32) ? 4 : 2;
+  if (row_elems <= 0) row_elems = cols;
   const cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)L, (cuuint64_t)B};
-  const cuuint64_t strides[2] = {(cuuint64_t)cols * es, (cuuint64_t)cols * es * (cuuint64_t)L};
-  const cuuint32_t box[3] = {32u, (cuuint32_t)rows, 1u};
+  const cuuint64_t strides[2] = {(cuuint64_t)row_elems * es, (cuuint64_t)row_elems * es * (cuuint64_t)L};
+  const cuuint32_t box[3] = {box_cols, (cuuint32_t)rows, 1u};
   const cuuint32_t estr[3] = {1u, 1u, 1u};
   const CUresult r = enc(map, io == BLR_F32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                          3, const_cast<void*>(base), dims, strides, box, estr,
@@ -190,33 +194,113 @@ blr_status launch_cooperative(K kernel, unsigned grid, int threads, size_t smem,
   return cuda_check(cudaLaunchKernelEx(&cfg, kernel, args), what);
 }
 
-// Grid of a warp-chain kernel: one warp per (batch row, channel group),
-// four warps per block.
-unsigned chain_grid(const Plan& p) {
-  const int64_t warps = p.B * ((p.D + 4 * p.nvl - 1) / (4 * p.nvl));
-  return (unsigned)((warps + 3) / 4);
+// ----------------------------------------------------------- serial kernels
+//
+// One warp per block, one block per chain. The ring's stage count is sized so
+// that the blocks that share an SM (chains / SMs of them) fit its shared memory.
+
+int sm_count() {
+  static std::mutex m;
+  static int counts[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  std::lock_guard<std::mutex> lock(m);
+  if (counts[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    counts[dev] = n;
+  }
+  return counts[dev];
 }
 
-template <typename T, class M>
-blr_status launch_chain_fwd(const blr::ChainFwdArgs& a, cudaStream_t st) {
-  const unsigned grid = chain_grid(a.p);
-  switch (a.p.nvl) {
-    case 8: blr::chain_fwd_kernel<T, M, 8><<<grid, 128, 0, st>>>(a); break;
-    case 4: blr::chain_fwd_kernel<T, M, 4><<<grid, 128, 0, st>>>(a); break;
-    default: blr::chain_fwd_kernel<T, M, 2><<<grid, 128, 0, st>>>(a); break;
-  }
-  return cuda_check(cudaGetLastError(), "launch chain_fwd_kernel");
+int seq_stages(int64_t n_chain, size_t stage_bytes) {
+  constexpr size_t kBudget = 200u << 10;  // shared memory per SM given to the rings
+  int64_t per_sm = (n_chain + sm_count() - 1) / sm_count();
+  if (per_sm < 1) per_sm = 1;
+  if (per_sm > 32) per_sm = 32;  // blocks per SM at most
+  int64_t s = (int64_t)(kBudget / (size_t)per_sm / stage_bytes);
+  if (s < 2) s = 2;
+  if (s > blr::kSeqMaxStages) s = blr::kSeqMaxStages;
+  return (int)s;
 }
 
-template <typename T, class M>
-blr_status launch_chain_bwd(const blr::ChainBwdArgs& a, cudaStream_t st) {
-  const unsigned grid = chain_grid(a.p);
-  switch (a.p.nvl) {
-    case 8: blr::chain_bwd_kernel<T, M, 8><<<grid, 128, 0, st>>>(a); break;
-    case 4: blr::chain_bwd_kernel<T, M, 4><<<grid, 128, 0, st>>>(a); break;
-    default: blr::chain_bwd_kernel<T, M, 2><<<grid, 128, 0, st>>>(a); break;
-  }
-  return cuda_check(cudaGetLastError(), "launch chain_bwd_kernel");
+template <typename K>
+blr_status allow_smem(K kernel, size_t smem) {
+  if (smem <= (48u << 10)) return BLR_OK;
+  return cuda_check(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                    "set dynamic shared memory size");
+}
+
+template <typename T, class M, int VEC, int R, int RB>
+blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
+  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB>;
+  a.stages = seq_stages(a.p.n_chain, 3 * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, 3);
+  BLR_TRY(allow_smem(kernel, smem));
+  kernel<<<(unsigned)a.p.n_chain, 32, smem, st>>>(a);
+  return cuda_check(cudaGetLastError(), "launch seq_fwd_kernel");
+}
+
+template <typename T, class M, int VEC, int R, int RB>
+blr_status launch_seq_bwd(blr::SeqBwdArgs& a, cudaStream_t st) {
+  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB>;
+  a.stages = seq_stages(a.p.n_chain, 4 * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, 4);
+  BLR_TRY(allow_smem(kernel, smem));
+  kernel<<<(unsigned)a.p.n_chain, 32, smem, st>>>(a);
+  return cuda_check(cudaGetLastError(), "launch seq_bwd_kernel");
+}
+
+// The serial kernels' views: x-shaped tensors as (D, L, B); gate_logits-shaped
+// ones as two (D, L, B) views of row length 2D, at column 0 (rho) and D (iota).
+blr_status seq_maps_x(CUtensorMap* m, const void* base, const Plan& plan, int rows) {
+  return make_tensor_map(m, base, plan.io, plan.D, plan.L, plan.B, rows, 32u * (uint32_t)plan.sv);
+}
+blr_status seq_maps_gl(CUtensorMap* mr, CUtensorMap* mi, const void* base, const Plan& plan, int rows) {
+  const size_t es = plan.io == BLR_F32 ? 4 : 2;
+  const uint32_t cols = 32u * (uint32_t)plan.sv;
+  BLR_TRY(make_tensor_map(mr, base, plan.io, plan.D, plan.L, plan.B, rows, cols, 2 * plan.D));
+  return make_tensor_map(mi, static_cast<const unsigned char*>(base) + (size_t)plan.D * es, plan.io,
+                         plan.D, plan.L, plan.B, rows, cols, 2 * plan.D);
+}
+
+blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const float* lambda,
+                        const float* h0, void* h, float* h_last, unsigned char* w, cudaStream_t st) {
+  blr::SeqFwdArgs a;
+  BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.sr));
+  BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, plan.sr));
+  a.write_h = h != nullptr;
+  if (a.write_h) BLR_TRY(seq_maps_x(&a.tm_h, h, plan, plan.sr));
+  else memset(&a.tm_h, 0, sizeof(a.tm_h));
+  a.p = plan;
+  a.lambda = lambda;
+  a.h0 = h0;
+  a.h_last = h_last;
+  a.ws = w;
+  a.stages = 2;
+  if (plan.io == BLR_F32) return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16>(a, st);
+  return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8>(a, st);
+}
+
+blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, const void* x,
+                        const void* gl, const float* lambda, const float* h0, void* dx, void* dgl,
+                        float* dlambda, float* dh0, unsigned char* w, cudaStream_t st) {
+  blr::SeqBwdArgs a;
+  BLR_TRY(seq_maps_x(&a.tm_dh, dh, plan, plan.srb));
+  BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.srb));
+  BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, plan.srb));
+  BLR_TRY(seq_maps_x(&a.tm_dx, dx, plan, plan.srb));
+  BLR_TRY(seq_maps_gl(&a.tm_dr, &a.tm_di, dgl, plan, plan.srb));
+  a.p = plan;
+  a.dh_last = dh_last;
+  a.lambda = lambda;
+  a.h0 = h0;
+  a.dlambda = dlambda;
+  a.dh0 = dh0;
+  a.ws = w;
+  a.stages = 2;
+  if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16>(a, st);
+  return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8>(a, st);
 }
 
 // Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
@@ -272,13 +356,8 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
-  if (plan.chain) {  // warp chains: no look-back records to empty
-    BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), nullptr, 0,
-                        reinterpret_cast<float*>(w + plan.off_k), lambda, desc->D, desc->c, st));
-    const blr::ChainFwdArgs ca{plan, x, gate_logits, h0, h, h_last, w};
-    if (desc->io == BLR_F32) return launch_chain_fwd<float, blr::MathPrecise>(ca, st);
-    return launch_chain_fwd<__nv_bfloat16, blr::MathFast>(ca, st);
-  }
+  if (plan.seq)  // serial kernels: no preparation
+    return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st);
   // Clear the forward header (counters, error word), empty the
   // forward records, precompute k = -c softplus(Lambda).
   BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fpre,
@@ -340,14 +419,9 @@ blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_la
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
-  if (plan.chain) {  // warp chains: clear the counters and partial sums only
-    BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, nullptr, 0,
-                        reinterpret_cast<float*>(w + plan.off_k), lambda, desc->D, desc->c, st));
-    const blr::ChainBwdArgs ca{plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
-                               dlambda, dh0, w};
-    if (desc->io == BLR_F32) return launch_chain_bwd<float, blr::MathPrecise>(ca, st);
-    return launch_chain_bwd<__nv_bfloat16, blr::MathFast>(ca, st);
-  }
+  if (plan.seq)  // the forward cleared the counters and partial sums
+    return scan_bwd_seq(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
+                        dh0, w, st);
   // Clear the backward header and the dLambda partial sums, empty the backward
   // records (the forward's records stay: they hold the carries).
   BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, w + plan.off_bagg,

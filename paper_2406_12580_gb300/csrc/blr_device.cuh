@@ -79,6 +79,57 @@ struct Io<__nv_bfloat16, 4> {  // 8 bytes
   }
 };
 
+template <>
+struct Io<float, 1> {  // 4 bytes
+  using T = float;
+  using Raw = float;
+  static constexpr int VEC = 1;
+  static __device__ __forceinline__ void unpack(const Raw& t, float (&v)[1]) { v[0] = t; }
+  static __device__ __forceinline__ void store(T* p, const float (&v)[1]) { __stcs(p, v[0]); }
+  static __device__ __forceinline__ void store_smem(unsigned char* p, const float (&v)[VEC]) {
+    *reinterpret_cast<float*>(p) = v[0];
+  }
+};
+
+template <>
+struct Io<float, 2> {  // 8 bytes
+  using T = float;
+  using Raw = float2;
+  static constexpr int VEC = 2;
+  static __device__ __forceinline__ void unpack(const Raw& t, float (&v)[2]) {
+    v[0] = t.x; v[1] = t.y;
+  }
+  static __device__ __forceinline__ void store(T* p, const float (&v)[2]) {
+    __stcs(reinterpret_cast<float2*>(p), make_float2(v[0], v[1]));
+  }
+  static __device__ __forceinline__ void store_smem(unsigned char* p, const float (&v)[VEC]) {
+    *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+  }
+};
+
+template <>
+struct Io<__nv_bfloat16, 2> {  // 4 bytes
+  using T = __nv_bfloat16;
+  using Raw = uint32_t;
+  static constexpr int VEC = 2;
+  static __device__ __forceinline__ void unpack(const Raw& t, float (&v)[2]) {
+    v[0] = __uint_as_float(t << 16); v[1] = __uint_as_float(t & 0xffff0000u);
+  }
+  static __device__ __forceinline__ void store(T* p, const float (&v)[2]) {
+    __stcs(reinterpret_cast<unsigned int*>(p), pack_bf16x2(v[0], v[1]));
+  }
+  static __device__ __forceinline__ void store_smem(unsigned char* p, const float (&v)[VEC]) {
+    *reinterpret_cast<uint32_t*>(p) = pack_bf16x2(v[0], v[1]);
+  }
+  // v = t / 2, halved on the packed pair (exact: an exponent decrement).
+  static __device__ __forceinline__ void unpack_half(const Raw& t, float (&v)[2]) {
+    uint32_t u;
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(u) : "r"(t), "r"(0x3f003f00u));  // (0.5, 0.5)
+    v[0] = __uint_as_float(u << 16);
+    v[1] = __uint_as_float(u & 0xffff0000u);
+  }
+};
+
 template <int N>
 __device__ __forceinline__ void load_f32(const float* p, float (&v)[N]) {
 #pragma unroll
@@ -205,6 +256,62 @@ struct MathFast {
   }
 };
 
+// ------------------------------------------------- per-element gate terms
+//
+// The serial kernels evaluate the gates of one element with as few
+// instructions as the precision policy allows. With l = k r = log(alpha) and
+// E = e^l - 1 (so alpha = 1 + E and 1 - alpha^2 = -E (2 + E)):
+//   decay_log(rho): l. MathFast folds sigmoid(rho) = (1 + tanh(rho/2)) / 2 into
+//     l = kh tanh(rho/2) + kh with kh = k/2 (one multiply-add after tanh).
+//   expm1<POLY>(l): the policy's Taylor series when every l of the channel lies
+//     in (-kExpm1Series, 0] (POLY), else the series or ex2 - 1 beyond it.
+constexpr float kExpm1Series = 0.25f;
+
+template <int DEG, bool POLY>
+__device__ __forceinline__ float expm1_neg(float l) {
+  const float e = expm1_taylor<DEG>(l);
+  if (POLY) return e;
+  return l > -kExpm1Series ? e : ex2_approx(l * 1.4426950408889634f) - 1.0f;
+}
+
+struct GatesPrecise : MathPrecise {
+  static constexpr int kDeg = 6;
+  static constexpr bool kHalfInputs = false;
+  static __device__ __forceinline__ float decay_log(float rho, float k, float) {
+    return k * sigmoid(rho);
+  }
+};
+
+struct GatesFast : MathFast {
+  static constexpr int kDeg = 4;
+  // With rho/2, iota/2 and x/2 at hand (halved on packed bfloat16 pairs):
+  // l = kh tanh(rho/2) + kh and i x = (x/2) tanh(iota/2) + x/2.
+  static constexpr bool kHalfInputs = true;
+  static __device__ __forceinline__ float decay_log_half(float hrho, float kh) {
+    return fmaf(kh, tanh_approx(hrho), kh);
+  }
+  static __device__ __forceinline__ float gated_x_half(float hiota, float hx) {
+    return fmaf(hx, tanh_approx(hiota), hx);
+  }
+  static __device__ __forceinline__ float sigmoid_half(float hz) {  // sigmoid(2 hz)
+    return fmaf(0.5f, tanh_approx(hz), 0.5f);
+  }
+  static __device__ __forceinline__ float decay_log(float rho, float, float kh) {
+    return fmaf(kh, tanh_approx(0.5f * rho), kh);
+  }
+};
+
+template <class G>
+struct GatePolicy;
+template <>
+struct GatePolicy<MathPrecise> {
+  using type = GatesPrecise;
+};
+template <>
+struct GatePolicy<MathFast> {
+  using type = GatesFast;
+};
+
 // k = -c softplus(Lambda), softplus(z) = max(z, 0) + log1p(exp(-|z|)), accurate.
 __device__ __forceinline__ float decay_rate(float c, float lambda) {
   return -c * (fmaxf(lambda, 0.0f) + log1pf(expf(-fabsf(lambda))));
@@ -320,13 +427,27 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// The same test, letting the hardware suspend the thread for up to
+// `hint_ns` while the phase is incomplete (instead of returning at once).
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+constexpr uint32_t kMbarSleepNs = 20000;  // per test; the whole wait stays bounded below
+
 // Waits for the stage's loads to land. Bounded: after the limit the block
 // records kErrTimeout and goes on with whatever the stage holds.
 __device__ __forceinline__ void mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* err) {
-  if (mbar_try_wait(bar, parity)) return;
+  if (mbar_try_wait_sleep(bar, parity, kMbarSleepNs)) return;
   const uint64_t start = global_timer_ns();
   for (uint32_t iter = 0;; ++iter) {
-    if (mbar_try_wait(bar, parity)) return;
+    if (mbar_try_wait_sleep(bar, parity, kMbarSleepNs)) return;
     if ((iter & 15u) == 15u && (global_timer_ns() - start > kWaitTimeoutNs || iter > kMaxWaitIters)) {
       atomicOr(err, kErrTimeout);
       return;
@@ -343,5 +464,27 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, uint64_
       "l"(tmap), "r"(c0), "r"(c1), "r"(c2), "r"(smem_addr(bar))
       : "memory");
 }
+
+// One 3-D tile store: shared memory into the box at (c0, c1, c2) of the tensor
+// map; elements outside the tensor are not written. The writes of the box in
+// shared memory must be fenced to the async proxy first.
+__device__ __forceinline__ void tma_store_3d(const void* tmap, const void* src, int c0, int c1,
+                                             int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(tmap),
+      "r"(smem_addr(src)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// Waits until at most N committed store groups still read shared memory.
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// Waits until every committed store group has completed.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 }  // namespace blr

@@ -60,21 +60,22 @@ struct BwdHeader {     // cleared before every backward
 inline int fwd_vec(int) { return 4; }
 inline int bwd_vec(int) { return 4; }
 
-// Problems with at least this many (batch row, channel group) chains, each at
-// most kChainMaxBlocks blocks long, use the warp-chain kernels (one warp walks
-// one chain); the others the tiled look-back kernels. The choice depends only
-// on the problem's shape.
-constexpr int64_t kChainMinWarps = 2048;
-constexpr int64_t kChainMaxBlocks = 16;
+// Problems with at least this many chains of 128-byte row segments (32
+// float32 or 64 bfloat16 channels of one batch row) use the serial kernels:
+// one warp walks one chain through the whole sequence. The others use the
+// tiled look-back kernels. The choice depends only on the problem's shape.
+constexpr int64_t kSeqMinChains = 256;
 
 struct Plan {
   int64_t B, L, D;
   int io;           // 0 = float32, 1 = bfloat16
   float c;
-  int chain;        // 1: warp-chain kernels, 0: tiled look-back kernels
-  int nvl;          // warp-chain: lanes along channels (chain width 4 * nvl channels)
-  int64_t bs;       // warp-chain: time steps per block = (32 / nvl) * kTc
-  int64_t n_blk;    // warp-chain: blocks per sequence
+  int seq;          // 1: serial kernels, 0: tiled look-back kernels
+  int sv;           // serial: channels per lane (row segment of 32 * sv channels)
+  int rb;           // serial: steps between the forward's kept states
+  int sr, srb;      // serial: rows per TMA box, forward and backward (multiples of rb)
+  int64_t n_chain;  // serial: chains = B * ceil(D / (32 * sv))
+  int64_t n_carry;  // serial: kept states per chain = ceil(L / rb) - 1
   int nwarps;       // warps per block = time sub-tiles per tile
   int64_t tsteps;   // time steps per tile = nwarps * kWarpSteps
   int64_t n_t;      // time tiles
@@ -131,24 +132,19 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   __builtin_memcpy(&cbits, &c, 4);
   h = fnv1a(h, cbits);
   p->tag = h | 1u;  // never 0, the value of a cleared header
-  p->chain = 0;
-  p->nvl = 8;
-  for (int nvl = 8; nvl >= 2; nvl >>= 1) {
-    const int64_t warps = B * ((D + 4 * nvl - 1) / (4 * nvl));
-    const int64_t bs = (int64_t)(32 / nvl) * kTc;
-    if (warps >= kChainMinWarps && (L + bs - 1) / bs <= kChainMaxBlocks) {
-      p->chain = 1;
-      p->nvl = nvl;
-      break;
-    }
-  }
-  p->bs = (int64_t)(32 / p->nvl) * kTc;
-  p->n_blk = (L + p->bs - 1) / p->bs;
-  // The forward's states after each time tile (or after each chain block but
-  // the last) are kept for the backward; the tiled kernels also need aggregates
-  // and backward records.
-  const size_t rec = (size_t)(p->chain ? p->n_blk - 1 : p->n_t) * (size_t)B * (size_t)D;
-  const size_t rec_t = p->chain ? 0 : rec;
+  p->sv = io == 0 ? 1 : 2;
+  p->rb = io == 0 ? 16 : 8;
+  p->sr = 16;
+  p->srb = io == 0 ? 16 : 8;
+  p->n_chain = B * ((D + 32 * p->sv - 1) / (32 * p->sv));
+  p->n_carry = (L + p->rb - 1) / p->rb - 1;
+  p->seq = p->n_chain >= kSeqMinChains ? 1 : 0;
+  // The forward's states after each time tile (or every rb steps of a serial
+  // chain, but the last) are kept for the backward; the tiled kernels also
+  // need aggregates and backward records.
+  const int64_t kept = p->seq ? p->n_carry : p->n_t;
+  const size_t rec = (size_t)kept * (size_t)B * (size_t)D;
+  const size_t rec_t = p->seq ? 0 : rec;
   size_t o = 0;
   p->off_fhdr = o;
   o = align_up(o + sizeof(FwdHeader), kAlign);

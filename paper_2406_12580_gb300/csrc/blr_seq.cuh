@@ -1,0 +1,532 @@
+// Serial scan kernels: the BD-LRU scan when a problem has enough independent
+// (batch row, channel group) chains to fill the GPU by itself.
+//
+// One warp (one thread block) owns CHW = 32 * VEC consecutive channels of one
+// batch row, a 128-byte row segment, and walks the whole sequence: each lane
+// runs the recurrence h_t = alpha_t h_{t-1} + beta_t x_t of Sec. 3.2 serially
+// for its VEC channels, one multiply-add per element, with the state in
+// registers. There is no cross-lane or cross-block combine and no second pass.
+//
+// Data movement is TMA both ways. The inputs stream through a ring of
+// shared-memory stages, one box of R rows per tensor; each lane writes
+// its outputs over its own, already consumed, inputs in the stage, and one TMA
+// store per output tensor sends the stage's outputs to global memory, clipped
+// to the tensor's extent (sequence and channel tails need no masking). A stage
+// is refilled at the start of the next iteration, once its store has read it,
+// so two stages already double-buffer.
+//
+// The forward also keeps the state after every RB steps, which the backward
+// uses as its starting points: the backward walks the sequence from the end in
+// sub-blocks of RB steps, recomputes the sub-block's gates and states forward
+// from the kept state (holding E = alpha - 1, 1 / sqrt(1 - alpha^2) and
+// h_{t-1} per element in registers), then runs the reverse recurrence
+// g_t = dh_t + alpha_{t+1} g_{t+1} through it, writing dx, d rho and d iota and
+// accumulating d Lambda.
+//
+// The forward's first block also restarts the workspace bookkeeping (error
+// word, problem tag, the backward's exit counter and d Lambda partial sums), so
+// no preparation kernel runs before either scan.
+#pragma once
+
+#include "blr_kernels.cuh"
+
+namespace blr {
+
+constexpr int kSeqMaxStages = 8;   // ring stages per warp
+
+// Tensor maps: (channels, time, batch) views with boxes of 32 * VEC channels x
+// R steps x 1 row. gate_logits is seen as two views of D channels each
+// (rho: columns [0, D), iota: columns [D, 2D)), so that boxes clip at D.
+struct SeqFwdArgs {
+  CUtensorMap tm_x;
+  CUtensorMap tm_r;
+  CUtensorMap tm_i;
+  CUtensorMap tm_h;  // unused when h is NULL
+  Plan p;
+  const float* lambda;
+  const float* h0;
+  float* h_last;
+  unsigned char* ws;
+  int stages;
+  int write_h;
+};
+
+struct SeqBwdArgs {
+  CUtensorMap tm_dh;
+  CUtensorMap tm_x;
+  CUtensorMap tm_r;
+  CUtensorMap tm_i;
+  CUtensorMap tm_dx;
+  CUtensorMap tm_dr;
+  CUtensorMap tm_di;
+  Plan p;
+  const float* dh_last;
+  const float* lambda;
+  const float* h0;
+  float* dlambda;
+  float* dh0;
+  unsigned char* ws;
+  int stages;
+};
+
+__device__ __forceinline__ unsigned char* align128(unsigned char* p) {
+  const uint32_t a = smem_addr(p);
+  return p + (((a + 127u) & ~127u) - a);
+}
+
+// Dynamic shared memory of a serial kernel: `stages` stages of NB boxes, one
+// mbarrier per stage, and slack for the 128-byte alignment of the boxes.
+template <typename T, int VEC, int R>
+__host__ __device__ constexpr uint32_t seq_box_bytes() {
+  return (uint32_t)(R * 32 * VEC * sizeof(T));
+}
+template <typename T, int VEC, int R>
+inline size_t seq_smem_bytes(int stages, int nb) {
+  return (size_t)stages * nb * seq_box_bytes<T, VEC, R>() + (size_t)stages * sizeof(uint64_t) + 128;
+}
+
+// Per-lane channel constants: k = -c softplus(Lambda), kh = k / 2, and whether
+// every channel of the warp keeps l = k r inside the series' range.
+template <int VEC>
+__device__ __forceinline__ bool seq_rates(const float* lambda, float c, int64_t d0, bool ch_ok,
+                                          float (&k)[VEC], float (&kh)[VEC]) {
+  bool poly = true;
+#pragma unroll
+  for (int v = 0; v < VEC; ++v) {
+    k[v] = ch_ok ? decay_rate(c, lambda[d0 + v]) : 0.0f;
+    kh[v] = 0.5f * k[v];
+    poly = poly && k[v] >= -kExpm1Series;
+  }
+  return __all_sync(kFull, poly);
+}
+
+// The ring: stage i holds NB boxes, then the S mbarriers. Block-uniform
+// bookkeeping of which stage holds which box and when it may be refilled.
+template <int NB, uint32_t BOX>
+struct SeqRing {
+  unsigned char* base;
+  uint64_t* bars;
+  int S;
+  __device__ __forceinline__ unsigned char* stage(int st) const { return base + (size_t)st * NB * BOX; }
+};
+
+// ------------------------------------------------------------------ forward
+
+// One stage, rows [0, rows) (all R when FULL). Phase 1 evaluates the
+// gates of every row (independent work), phase 2 runs the recurrence and
+// writes h over x in the stage. `cidx` is the index of the next kept state.
+template <class IO, class G, bool POLY, bool FULL, int R, int RB>
+__device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
+                                              const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
+                                              float (&hc)[IO::VEC], float* carry, int64_t& cidx,
+                                              int64_t n_carry, int64_t BD, bool ch_ok) {
+  using Raw = typename IO::Raw;
+  constexpr int V = IO::VEC;
+  constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
+  constexpr uint32_t BOX = R * ROWB;
+  float al[R][V], uu[R][V];
+#pragma unroll
+  for (int s = 0; s < R; ++s) {
+    if (FULL || s < rows) {
+      float xv[V], rv[V], iv[V];
+      if constexpr (G::kHalfInputs) {
+        IO::unpack_half(*reinterpret_cast<const Raw*>(sb + s * ROWB), xv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(sb + BOX + s * ROWB), rv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(sb + 2 * BOX + s * ROWB), iv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          const float e = expm1_neg<G::kDeg, POLY>(G::decay_log_half(rv[v], kh[v]));
+          al[s][v] = 1.0f + e;
+          uu[s][v] = G::sqrt(-e * (e + 2.0f)) * G::gated_x_half(iv[v], xv[v]);
+        }
+      } else {
+        IO::unpack(*reinterpret_cast<const Raw*>(sb + s * ROWB), xv);
+        IO::unpack(*reinterpret_cast<const Raw*>(sb + BOX + s * ROWB), rv);
+        IO::unpack(*reinterpret_cast<const Raw*>(sb + 2 * BOX + s * ROWB), iv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          const float e = expm1_neg<G::kDeg, POLY>(G::decay_log(rv[v], k[v], kh[v]));
+          al[s][v] = 1.0f + e;
+          uu[s][v] = G::sqrt(-e * (e + 2.0f)) * (G::sigmoid(iv[v]) * xv[v]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int s = 0; s < R; ++s) {
+    if (FULL || s < rows) {
+      float out[V];
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        hc[v] = fmaf(al[s][v], hc[v], uu[s][v]);
+        out[v] = hc[v];
+      }
+      IO::store_smem(sb + s * ROWB, out);
+      if ((s + 1) % RB == 0) {  // a kept state: after step (cidx + 1) RB - 1
+        if (cidx < n_carry && ch_ok) {
+#pragma unroll
+          for (int v = 0; v < V; ++v) carry[cidx * BD + v] = hc[v];
+        }
+        ++cidx;
+      }
+    }
+  }
+}
+
+template <typename T, class M, int VEC, int R, int RB>
+__global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ SeqFwdArgs a) {
+  using IO = Io<T, VEC>;
+  using G = typename GatePolicy<M>::type;
+  constexpr int CHW = 32 * VEC;
+  constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
+  static_assert(R % RB == 0, "kept states must fall on stage rows");
+  const Plan& p = a.p;
+  extern __shared__ unsigned char seq_smem[];
+  SeqRing<3, BOX> ring{align128(seq_smem), nullptr, a.stages};
+  ring.bars = reinterpret_cast<uint64_t*>(ring.stage(ring.S));
+
+  const int lane = threadIdx.x;
+  const int64_t n_g = (p.D + CHW - 1) / CHW;
+  const int64_t b = blockIdx.x / n_g;
+  const int64_t g = blockIdx.x - b * n_g;
+  const int64_t d0 = g * CHW + lane * VEC;
+  const bool ch_ok = d0 < p.D;  // D % 8 == 0: a lane's VEC channels are all in or all out
+  const int64_t BD = p.B * p.D;
+  FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
+  BwdHeader* bh = reinterpret_cast<BwdHeader*>(a.ws + p.off_bhdr);
+
+  if (blockIdx.x == 0) {
+    double* acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
+    for (int64_t i = lane; i < (int64_t)kStripes * p.D; i += 32) acc[i] = 0.0;
+    if (lane == 0) {
+      fh->err = 0u;
+      bh->exited = 0u;
+      fh->tag = p.tag;
+      fh->complete = 1u;
+    }
+  }
+
+  float k[VEC], kh[VEC], hc[VEC];
+  const bool poly = seq_rates<VEC>(a.lambda, p.c, d0, ch_ok, k, kh);
+#pragma unroll
+  for (int v = 0; v < VEC; ++v) hc[v] = (ch_ok && a.h0 != nullptr) ? a.h0[b * p.D + d0 + v] : 0.0f;
+
+  const int64_t nblk = (p.L + R - 1) / R;
+  const int cd = (int)(g * CHW), cb = (int)b;
+  auto issue = [&](int st, int64_t j) {
+    unsigned char* dst = ring.stage(st);
+    const int t = (int)(j * R);
+    mbar_arrive_expect_tx(&ring.bars[st], 3 * BOX);
+    tma_load_3d(dst, &a.tm_x, &ring.bars[st], cd, t, cb);
+    tma_load_3d(dst + BOX, &a.tm_r, &ring.bars[st], cd, t, cb);
+    tma_load_3d(dst + 2 * BOX, &a.tm_i, &ring.bars[st], cd, t, cb);
+  };
+  if (lane == 0) {
+    for (int s = 0; s < ring.S; ++s) mbar_init(&ring.bars[s], 1);
+    fence_mbar_init();
+    for (int s = 0; s < ring.S && s < nblk; ++s) issue(s, s);
+  }
+  __syncwarp();
+
+  float* carry = reinterpret_cast<float*>(a.ws + p.off_fpre) + b * p.D + d0;
+  int64_t cidx = 0;
+  const int64_t n_carry = p.n_carry;
+  int st = 0, prev = ring.S - 1;
+  uint32_t phase = 0;
+  for (int64_t j = 0; j < nblk; ++j) {
+    mbar_wait(&ring.bars[st], phase, &fh->err);
+    // the previous stage's store has read it by now (or shortly will): refill it
+    if (lane == 0 && j > 0 && j - 1 + ring.S < nblk) {
+      if (a.write_h) bulk_wait_read<0>();
+      issue(prev, j - 1 + ring.S);
+    }
+    unsigned char* sb = ring.stage(st);
+    unsigned char* lb = sb + lane * VEC * sizeof(T);
+    const int64_t left = p.L - j * R;
+    const int rows = (int)(left < R ? left : R);
+    if (rows == R) {
+      if (poly)
+        seq_fwd_stage<IO, G, true, true, R, RB>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
+      else
+        seq_fwd_stage<IO, G, false, true, R, RB>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
+    } else {
+      seq_fwd_stage<IO, G, false, false, R, RB>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
+    }
+    fence_proxy_async_smem();  // the stage's h rows, visible to the TMA store
+    __syncwarp();
+    if (lane == 0 && a.write_h) {
+      tma_store_3d(&a.tm_h, sb, cd, (int)(j * R), cb);
+      bulk_commit();
+    }
+    prev = st;
+    if (++st == ring.S) {
+      st = 0;
+      phase ^= 1u;
+    }
+  }
+  if (lane == 0 && a.write_h) bulk_wait_all();
+  if (a.h_last != nullptr && ch_ok) {
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) a.h_last[b * p.D + d0 + v] = hc[v];
+  }
+}
+
+// ----------------------------------------------------------------- backward
+
+// One sub-block of RB steps (rows [0, srows) when not FULL) starting at row
+// `row0` of the stage: forward recompute from the state hc, then the reverse
+// recurrence carrying w = alpha g. dx, d rho and d iota overwrite dh, rho and
+// iota of the same rows in the stage.
+template <class IO, class G, bool POLY, bool FULL, int R, int RB>
+__device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int srows,
+                                            const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
+                                            float (&hc)[IO::VEC], float (&w)[IO::VEC],
+                                            float (&dlr)[IO::VEC]) {
+  using Raw = typename IO::Raw;
+  constexpr int V = IO::VEC;
+  constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
+  constexpr uint32_t BOX = R * ROWB;
+  // boxes of a backward stage: dh, x, rho, iota
+  unsigned char* s_dh = lb + row0 * ROWB;
+  const unsigned char* s_x = s_dh + BOX;
+  unsigned char* s_r = s_dh + 2 * BOX;
+  unsigned char* s_i = s_dh + 3 * BOX;
+  float E[RB][V], RS[RB][V], HP[RB][V];
+#pragma unroll
+  for (int s = 0; s < RB; ++s) {
+    if (FULL || s < srows) {
+      float xv[V], rv[V], iv[V], ix[V], l[V];
+      if constexpr (G::kHalfInputs) {
+        IO::unpack_half(*reinterpret_cast<const Raw*>(s_x + s * ROWB), xv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(s_i + s * ROWB), iv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          l[v] = G::decay_log_half(rv[v], kh[v]);
+          ix[v] = G::gated_x_half(iv[v], xv[v]);
+        }
+      } else {
+        IO::unpack(*reinterpret_cast<const Raw*>(s_x + s * ROWB), xv);
+        IO::unpack(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
+        IO::unpack(*reinterpret_cast<const Raw*>(s_i + s * ROWB), iv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          l[v] = G::decay_log(rv[v], k[v], kh[v]);
+          ix[v] = G::sigmoid(iv[v]) * xv[v];
+        }
+      }
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        const float e = expm1_neg<G::kDeg, POLY>(l[v]);
+        const float q = -e * (e + 2.0f);
+        const float rs = rsqrt_approx(fmaxf(q, 1e-30f));  // 1/sqrt(q); finite at q = 0
+        E[s][v] = e;
+        RS[s][v] = rs;
+        HP[s][v] = hc[v];
+        hc[v] = fmaf(1.0f + e, hc[v], (q * rs) * ix[v]);
+      }
+    }
+  }
+#pragma unroll
+  for (int s = RB - 1; s >= 0; --s) {
+    if (FULL || s < srows) {
+      float gv[V], xv[V], rv[V], iv[V], ox[V], orho[V], oiota[V];
+      IO::unpack(*reinterpret_cast<const Raw*>(s_dh + s * ROWB), gv);
+      IO::unpack(*reinterpret_cast<const Raw*>(s_x + s * ROWB), xv);
+      if constexpr (G::kHalfInputs) {
+        IO::unpack_half(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(s_i + s * ROWB), iv);
+      } else {
+        IO::unpack(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
+        IO::unpack(*reinterpret_cast<const Raw*>(s_i + s * ROWB), iv);
+      }
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        const float e = E[s][v], rs = RS[s][v];
+        const float alpha = 1.0f + e;
+        const float q = -e * (e + 2.0f);
+        float r, i;
+        if constexpr (G::kHalfInputs) {
+          r = G::sigmoid_half(rv[v]);
+          i = G::sigmoid_half(iv[v]);
+        } else {
+          r = G::sigmoid(rv[v]);
+          i = G::sigmoid(iv[v]);
+        }
+        const float g = gv[v] + w[v];
+        w[v] = alpha * g;
+        const float ix = i * xv[v];
+        const float u = (q * rs) * ix;
+        ox[v] = (g * (q * rs)) * i;
+        oiota[v] = (g * u) * (1.0f - i);
+        // d/dl of h_t: alpha g (h_{t-1} - alpha u / q), with alpha g = w and
+        // u / q = i x rs
+        const float dl = w[v] * (HP[s][v] - (alpha * rs) * ix);
+        orho[v] = (dl * k[v]) * fmaf(-r, r, r);
+        dlr[v] = fmaf(dl, r, dlr[v]);
+      }
+      IO::store_smem(s_dh + s * ROWB, ox);
+      IO::store_smem(s_r + s * ROWB, orho);
+      IO::store_smem(s_i + s * ROWB, oiota);
+    }
+  }
+}
+
+template <typename T, class M, int VEC, int R, int RB>
+__global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(const __grid_constant__ SeqBwdArgs a) {
+  using IO = Io<T, VEC>;
+  using G = typename GatePolicy<M>::type;
+  constexpr int CHW = 32 * VEC;
+  constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
+  constexpr int NSUB = R / RB;
+  static_assert(R % RB == 0, "sub-blocks must tile a stage");
+  const Plan& p = a.p;
+  extern __shared__ unsigned char seq_smem[];
+  SeqRing<4, BOX> ring{align128(seq_smem), nullptr, a.stages};
+  ring.bars = reinterpret_cast<uint64_t*>(ring.stage(ring.S));
+
+  const int lane = threadIdx.x;
+  FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
+  BwdHeader* bh = reinterpret_cast<BwdHeader*>(a.ws + p.off_bhdr);
+  {
+    int ok = 0;
+    if (lane == 0) {
+      ok = __ldcg(&fh->tag) == p.tag && __ldcg(&fh->complete) == 1u;
+      if (!ok) atomicOr(&fh->err, kErrWorkspace);
+    }
+    if (!__shfl_sync(kFull, ok, 0)) return;  // no forward states for this problem: write nothing
+  }
+  const int64_t n_g = (p.D + CHW - 1) / CHW;
+  const int64_t b = blockIdx.x / n_g;
+  const int64_t g = blockIdx.x - b * n_g;
+  const int64_t d0 = g * CHW + lane * VEC;
+  const bool ch_ok = d0 < p.D;
+  const int64_t BD = p.B * p.D;
+
+  float k[VEC], kh[VEC], w[VEC], dlr[VEC], nhc[VEC];
+  const bool poly = seq_rates<VEC>(a.lambda, p.c, d0, ch_ok, k, kh);
+#pragma unroll
+  for (int v = 0; v < VEC; ++v) {
+    w[v] = (ch_ok && a.dh_last != nullptr) ? a.dh_last[b * p.D + d0 + v] : 0.0f;
+    dlr[v] = 0.0f;
+  }
+  const float* carry = reinterpret_cast<const float*>(a.ws + p.off_fpre) + b * p.D + d0;
+  // the state before sub-block m: h0 for m = 0, else kept state m - 1
+  auto load_start = [&](int64_t m, float (&out)[VEC]) {
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+      out[v] = 0.0f;
+      if (ch_ok) {
+        if (m > 0)
+          out[v] = __ldcg(carry + (m - 1) * BD + v);
+        else if (a.h0 != nullptr)
+          out[v] = a.h0[b * p.D + d0 + v];
+      }
+    }
+  };
+
+  const int64_t nblk = (p.L + R - 1) / R;
+  const int cd = (int)(g * CHW), cb = (int)b;
+  auto issue = [&](int st, int64_t j) {
+    unsigned char* dst = ring.stage(st);
+    const int t = (int)(j * R);
+    mbar_arrive_expect_tx(&ring.bars[st], 4 * BOX);
+    tma_load_3d(dst, &a.tm_dh, &ring.bars[st], cd, t, cb);
+    tma_load_3d(dst + BOX, &a.tm_x, &ring.bars[st], cd, t, cb);
+    tma_load_3d(dst + 2 * BOX, &a.tm_r, &ring.bars[st], cd, t, cb);
+    tma_load_3d(dst + 3 * BOX, &a.tm_i, &ring.bars[st], cd, t, cb);
+  };
+  if (lane == 0) {
+    for (int s = 0; s < ring.S; ++s) mbar_init(&ring.bars[s], 1);
+    fence_mbar_init();
+    for (int s = 0; s < ring.S && s < nblk; ++s) issue(s, nblk - 1 - s);
+  }
+  __syncwarp();
+
+  int64_t m = (p.L + RB - 1) / RB - 1;  // the sub-block processed next
+  load_start(m, nhc);
+  int st = 0, prev = ring.S - 1;
+  uint32_t phase = 0;
+  for (int64_t i = 0; i < nblk; ++i) {
+    const int64_t j = nblk - 1 - i;
+    mbar_wait(&ring.bars[st], phase, &fh->err);
+    // the previous stage's stores have read it by now (or shortly will): refill it
+    if (lane == 0 && i > 0 && i - 1 + ring.S < nblk) {
+      bulk_wait_read<0>();
+      issue(prev, nblk - 1 - (i - 1 + ring.S));
+    }
+    unsigned char* sb = ring.stage(st);
+    unsigned char* lb = sb + lane * VEC * sizeof(T);
+    const int64_t left = p.L - j * R;
+    const int rows = (int)(left < R ? left : R);
+#pragma unroll
+    for (int q = NSUB - 1; q >= 0; --q) {
+      const int row0 = q * RB;
+      if (row0 < rows) {
+        const int srows = rows - row0 < RB ? rows - row0 : RB;
+        float hc[VEC];
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) hc[v] = nhc[v];
+        if (m > 0) load_start(m - 1, nhc);  // the next sub-block's start, in flight meanwhile
+        if (srows == RB) {
+          if (poly)
+            seq_bwd_sub<IO, G, true, true, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
+          else
+            seq_bwd_sub<IO, G, false, true, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
+        } else {
+          seq_bwd_sub<IO, G, false, false, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
+        }
+        --m;
+      }
+    }
+    fence_proxy_async_smem();  // the stage's outputs, visible to the TMA stores
+    __syncwarp();
+    if (lane == 0) {
+      const int t = (int)(j * R);
+      tma_store_3d(&a.tm_dx, sb, cd, t, cb);
+      tma_store_3d(&a.tm_dr, sb + 2 * BOX, cd, t, cb);
+      tma_store_3d(&a.tm_di, sb + 3 * BOX, cd, t, cb);
+      bulk_commit();
+    }
+    prev = st;
+    if (++st == ring.S) {
+      st = 0;
+      phase ^= 1u;
+    }
+  }
+  if (lane == 0) bulk_wait_all();
+
+  double* acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
+  if (ch_ok) {
+    if (a.dh0 != nullptr) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) a.dh0[b * p.D + d0 + v] = w[v];
+    }
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) atomicAdd(acc + (b % kStripes) * p.D + d0 + v, (double)dlr[v]);
+  }
+  // The last block out turns the partial sums into dLambda and clears them
+  // (and the exit counter) for the next backward.
+  __syncwarp();
+  int last = 0;
+  if (lane == 0) {
+    __threadfence();
+    last = atomicAdd(&bh->exited, 1u) == gridDim.x - 1;
+  }
+  if (__shfl_sync(kFull, last, 0)) {
+    __threadfence();
+    for (int64_t d = lane; d < p.D; d += 32) {
+      double sum = 0.0;
+      for (int s2 = 0; s2 < kStripes; ++s2) {
+        sum += __ldcg(&acc[s2 * p.D + d]);
+        acc[s2 * p.D + d] = 0.0;
+      }
+      const double lam = (double)a.lambda[d];
+      const double sig = 1.0 / (1.0 + exp(-lam));  // d softplus / d Lambda
+      a.dlambda[d] = (float)(-(double)p.c * sig * sum);
+    }
+    if (lane == 0) bh->exited = 0u;
+  }
+}
+
+}  // namespace blr
