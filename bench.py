@@ -77,6 +77,27 @@ def dist_env():
     return rank, world, local
 
 
+def rank_workload(cfg, rank: int):
+    """The workload rank `rank` scans in a multi-GPU run: the same shape with
+    its own seed (batch rows are independent problems, so ranks share no data
+    and need no collective on the data path). Rank 0 scans the workload itself."""
+    if rank == 0:
+        return cfg
+    return dataclasses.replace(cfg, seed=cfg.seed + 7919 * rank)
+
+
+def max_over_ranks(local: float, world: int, device=None) -> float:
+    """The largest of the ranks' values (the step time of the slowest rank);
+    `device` is where the reduction tensor lives (CUDA for NCCL, CPU for gloo)."""
+    if world == 1:
+        return local
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([local], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -337,6 +358,7 @@ def run_ours(args):
     cfg = I.CONFIGS[args.config]
     if args.seq_len > 0:
         cfg = dataclasses.replace(cfg, name=f"{cfg.name} at L={args.seq_len}", L=args.seq_len)
+    cfg = rank_workload(cfg, rank)
     inp = I.make_scan_inputs(cfg)
     buf = ScanBuffers.from_inputs(inp, device=dev)
     n = cfg.elements
@@ -379,10 +401,7 @@ def run_ours(args):
     clock_rows = sampler.stop()
 
     total_ms = sum(fwd_ms) + sum(bwd_ms)
-    t_local = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        torch.distributed.all_reduce(t_local, op=torch.distributed.ReduceOp.MAX)
-    t_max_ms = float(t_local.item())
+    t_max_ms = max_over_ranks(total_ms, world, device=dev)
     value = world * n * args.steps / (t_max_ms * 1e-3)
     summ = workload_summary(cfg, fwd_ms, bwd_ms, peak)
 
