@@ -32,11 +32,16 @@ SMALL = [
     dict(B=2, L=1031, D=256, decay=(0.99, 0.9999), random_h0=True, random_dh_last=True),
     dict(B=5, L=129, D=128, c=2.5, random_h0=True),
     dict(B=2, L=200, D=64, gate_std=3.0, x_std=4.0),
-    # enough (batch row, channel group) chains for the warp-chain kernels, at
-    # each chain width: 32 channels, 16 (with a partial group), 8
+    # enough (batch row, channel group) chains for the serial kernels, with
+    # partial channel groups and sequence tails
     dict(B=2100, L=5, D=32, random_h0=True, random_dh_last=True),
     dict(B=700, L=37, D=40, random_h0=True),
     dict(B=1100, L=130, D=16, random_dh_last=True, decay=(0.99, 0.9999)),
+    # serial chains split into time segments (2 or 4 warps per chain), with a
+    # short last segment, h0 and dh_last entering through the segment maps
+    dict(B=300, L=203, D=24, random_h0=True, random_dh_last=True),
+    dict(B=600, L=100, D=72, random_h0=True, random_dh_last=True),
+    dict(B=520, L=129, D=32, decay=(0.99, 0.9999)),
 ]
 
 
