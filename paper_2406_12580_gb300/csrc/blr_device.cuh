@@ -218,11 +218,8 @@ struct MathPrecise {
     if (l > -0.25f) return expm1_taylor<6>(l);
     return ex2_approx(l * 1.4426950408889634f) - 1.0f;
   }
-  static __device__ __forceinline__ float sqrt(float q) {
-    float n, inv_n;
-    sqrt_pair(q, n, inv_n);
-    return n;
-  }
+  // sqrt(q) for q >= 0 (one sqrt.approx; 0 at q = 0, denormals flushed)
+  static __device__ __forceinline__ float sqrt(float q) { return sqrt_approx(q); }
   // beta = sqrt(q) i, u = beta x and c2 = alpha u / q (= alpha i x / n).
   static __device__ __forceinline__ void norm_terms(float q, float i, float x, float alpha,
                                                     float& beta, float& u, float& c2) {
