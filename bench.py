@@ -35,6 +35,7 @@ sys.path.insert(0, ROOT)
 METRIC = "BD-LRU scan fwd+bwd elements/s and achieved HBM GB/s vs GB300 peak (1 GPU)"
 UNIT = "elements/s"
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0  # GB300 HBM3e nominal, reported beside the measured-peak fractions
 
 # Compulsory HBM bytes per element (inputs read once, outputs written once;
 # the per-tile carries and O(B*D) state are overhead, not counted):
@@ -434,6 +435,7 @@ def run_ours(args):
                    "inputs": "seeded synthetic (paper_2406_12580_gb300.inputs), resident in HBM"},
         "hbm_gbs": summ.get("fwd_bwd_gbs", summ["fwd_gbs"]),
         "hbm_frac": summ.get("fwd_bwd_frac", summ["fwd_frac"]),
+        "hbm_frac_nominal": summ.get("fwd_bwd_gbs", summ["fwd_gbs"]) / NOMINAL_HBM_GBS,
         "roofline": roofline,
         "gpu_launches": (1 if cfg.fwd_only else 2) * per_call * args.steps,
         "wall_s_timed_region": wall,
@@ -523,7 +525,51 @@ def other_workloads(flush, peak, dev, headline):
         out[f"step_{io}"] = {"workload": scfg.name, "ms": ms,
                              "elements_per_s": scfg.elements / (ms * 1e-3), "gbs": gbs,
                              "frac": gbs / peak}
+        del sbuf
+    out["step_f32_graph"] = step_graph(flush, peak, dev)
     return out
+
+
+def step_graph(flush, peak, dev, n_tok=8, reps=20):
+    """Recurrent serving: n_tok consecutive steps h <- step(h, x_k, gate_logits_k)
+    with distinct inputs per step (n_tok x 84 MB, more than L2), launched back to
+    back from one CUDA graph; L2 flushed before each replay."""
+    import torch
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import StepBuffers
+    bufs = [StepBuffers.from_inputs(I.make_step_inputs(
+        I.StepConfig(f"recurrent step B=65536 D=64 f32 token {k}", 65536, 64, "f32", seed=100 + k)),
+        device=dev) for k in range(n_tok)]
+    h = [bufs[0].h_prev, torch.empty_like(bufs[0].h_prev)]
+
+    def run():
+        for k, b in enumerate(bufs):
+            b.h_prev, b.h_t = h[k % 2], h[(k + 1) % 2]
+            b.step()
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        run()  # warm-up outside capture
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        run()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps)]
+    for e0, e1 in ev:
+        flush()
+        e0.record()
+        g.replay()
+        e1.record()
+    torch.cuda.synchronize()
+    ms = statistics.median(a.elapsed_time(b) for a, b in ev[3:]) / n_tok
+    el = bufs[0].B * bufs[0].D
+    gbs = el * step_bytes_per_elem("f32") / (ms * 1e-3) / 1e9
+    return {"workload": f"{n_tok} recurrent steps B=65536 D=64 f32 in one CUDA graph",
+            "ms_per_step": ms, "elements_per_s": el / (ms * 1e-3), "gbs": gbs, "frac": gbs / peak}
 
 
 def main():

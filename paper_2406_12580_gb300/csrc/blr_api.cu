@@ -278,7 +278,10 @@ blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const f
   a.h_last = h_last;
   a.ws = w;
   a.stages = 2;
-  if (plan.io == BLR_F32) return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16>(a, st);
+  if (plan.io == BLR_F32) {
+    if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16>(a, st);
+    return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16>(a, st);
+  }
   return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8>(a, st);
 }
 

@@ -65,6 +65,7 @@ inline int bwd_vec(int) { return 4; }
 // one warp walks one chain through the whole sequence. The others use the
 // tiled look-back kernels. The choice depends only on the problem's shape.
 constexpr int64_t kSeqMinChains = 256;
+constexpr int64_t kSeqTallRowsMinL = 1024;
 
 struct Plan {
   int64_t B, L, D;
@@ -134,7 +135,10 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   p->tag = h | 1u;  // never 0, the value of a cleared header
   p->sv = io == 0 ? 1 : 2;
   p->rb = io == 0 ? 16 : 8;
-  p->sr = 16;
+  // Long float32 sequences stream the forward in 32-row boxes (fewer, larger
+  // TMA loads per chain); shorter ones in 16-row boxes, which reach the first
+  // rows sooner.
+  p->sr = (io == 0 && L >= kSeqTallRowsMinL) ? 32 : 16;
   p->srb = io == 0 ? 16 : 8;
   p->n_chain = B * ((D + 32 * p->sv - 1) / (32 * p->sv));
   p->n_carry = (L + p->rb - 1) / p->rb - 1;

@@ -46,6 +46,9 @@ SMALL = [
     # the general e^l - 1 branch) and c != 1, on both kernel families
     dict(B=3, L=150, D=40, decay=(0.05, 0.95), c=3.0, random_h0=True, random_dh_last=True),
     dict(B=400, L=90, D=40, decay=(0.05, 0.95), c=0.5, random_h0=True, random_dh_last=True),
+    # a long sequence with many chains (float32: the forward's 32-row boxes),
+    # ending in a partial box
+    dict(B=260, L=1100, D=8, decay=(0.99, 0.9999), random_h0=True, random_dh_last=True),
 ]
 
 
