@@ -403,7 +403,10 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   const bool ch_ok = d0 < p.D;
   const int64_t BD = p.B * p.D;
 
-  float k[VEC], kh[VEC], w[VEC], dlr[VEC], nhc[VEC];
+  // The start states of the next QD sub-blocks, loaded QD sub-blocks ahead of
+  // use (one ahead for bfloat16, whose registers are fully used).
+  constexpr int QD = sizeof(T) == 4 ? 4 : 1;
+  float k[VEC], kh[VEC], w[VEC], dlr[VEC], sq[QD][VEC];
   const bool poly = seq_rates<VEC>(a.lambda, p.c, d0, ch_ok, k, kh);
 #pragma unroll
   for (int v = 0; v < VEC; ++v) {
@@ -444,7 +447,12 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   __syncwarp();
 
   int64_t m = (p.L + RB - 1) / RB - 1;  // the sub-block processed next
-  load_start(m, nhc);
+#pragma unroll
+  for (int u = 0; u < QD; ++u) {
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) sq[u][v] = 0.0f;
+    if (m - u >= 0) load_start(m - u, sq[u]);
+  }
   int st = 0, prev = ring.S - 1;
   uint32_t phase = 0;
   for (int64_t i = 0; i < nblk; ++i) {
@@ -466,8 +474,13 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
         const int srows = rows - row0 < RB ? rows - row0 : RB;
         float hc[VEC];
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) hc[v] = nhc[v];
-        if (m > 0) load_start(m - 1, nhc);  // the next sub-block's start, in flight meanwhile
+        for (int v = 0; v < VEC; ++v) hc[v] = sq[0][v];
+#pragma unroll
+        for (int u = 0; u + 1 < QD; ++u) {
+#pragma unroll
+          for (int v = 0; v < VEC; ++v) sq[u][v] = sq[u + 1][v];
+        }
+        if (m - QD >= 0) load_start(m - QD, sq[QD - 1]);  // in flight for QD sub-blocks
         if (srows == RB) {
           if (poly)
             seq_bwd_sub<IO, G, true, true, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
