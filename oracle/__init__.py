@@ -13,6 +13,8 @@ Functions and the passages they follow:
   fwd(x, gl, lam, h0, c)            -> h, h_last             Sec. 3.2, Eq. linrnn
   bwd(dh, x, gl, lam, h0, dh_last)  -> dx, dgl, dlam, dh0    chain rule of Sec. 3.2 (not printed in the paper)
   step(h_prev, x, gl, lam, c)       -> h_t                   Sec. 1 / Sec. 4.3 (recurrent inference)
+  fwd_gated(x, gl, lam, z, h0, c)   -> y = h SiLU(z), h_last  Alg. 1 (the scan, then the merge H_y (x) SiLU(H_z))
+  bwd_gated(dy, x, gl, lam, z, ...) -> dx, dgl, dlam, dh0, dz  chain rule through the merge, then bwd
 
 Every function is pinned by the CPU tests in ``tests/test_oracle_pins.py``
 (closed forms, special cases, brute force, the paper's two-tree scan,
@@ -93,8 +95,11 @@ class Oracle:
         lib.blr_oracle_bwd.argtypes = [_I64, _I64, _I64, ctypes.c_double, _P, _P, _P, _P, _P, _P,
                                        _P, _P, _P, _P, ctypes.c_int]
         lib.blr_oracle_step.argtypes = [_I64, _I64, ctypes.c_double, _P, _P, _P, _P, _P]
+        lib.blr_oracle_merge.argtypes = [_I64, _P, _P, _P]
+        lib.blr_oracle_merge_bwd.argtypes = [_I64, _P, _P, _P, _P, _P]
         lib.blr_oracle_has_openmp.restype = ctypes.c_int
-        for f in ("blr_oracle_gates", "blr_oracle_fwd", "blr_oracle_bwd", "blr_oracle_step"):
+        for f in ("blr_oracle_gates", "blr_oracle_fwd", "blr_oracle_bwd", "blr_oracle_step",
+                  "blr_oracle_merge", "blr_oracle_merge_bwd"):
             getattr(lib, f).restype = None
         self._lib = lib
         self.has_openmp = bool(lib.blr_oracle_has_openmp())
@@ -149,6 +154,35 @@ class Oracle:
         h_t = np.empty((B, D))
         self._lib.blr_oracle_step(B, D, c, _ptr(h_prev), _ptr(x), _ptr(gl), _ptr(lam), _ptr(h_t))
         return h_t
+
+    def merge(self, h, z):
+        """y = h SiLU(z), elementwise (Alg. 1, the merge of the two branches)."""
+        h = _f64(h)
+        z = _f64(z, h.shape)
+        y = np.empty(h.shape)
+        self._lib.blr_oracle_merge(h.size, _ptr(h), _ptr(z), _ptr(y))
+        return y
+
+    def merge_bwd(self, dy, h, z):
+        """(dh, dz) of the merge for the upstream gradient dy."""
+        h = _f64(h)
+        dy, z = _f64(dy, h.shape), _f64(z, h.shape)
+        dh, dz = np.empty(h.shape), np.empty(h.shape)
+        self._lib.blr_oracle_merge_bwd(h.size, _ptr(dy), _ptr(h), _ptr(z), _ptr(dh), _ptr(dz))
+        return dh, dz
+
+    def fwd_gated(self, x, gl, lam, z, h0=None, c: float = 1.0, threads: int = 1):
+        """The scan followed by the merge: (y, h_last), y = h SiLU(z)."""
+        h, h_last = self.fwd(x, gl, lam, h0, c=c, threads=threads)
+        return self.merge(h, z), h_last
+
+    def bwd_gated(self, dy, x, gl, lam, z, h0=None, dh_last=None, c: float = 1.0, threads: int = 1):
+        """Backward of fwd_gated for the loss sum dy y + sum dh_last h_last:
+        (dx, dgl, dlam, dh0, dz)."""
+        h, _ = self.fwd(x, gl, lam, h0, c=c, threads=threads)
+        dh, dz = self.merge_bwd(dy, h, z)
+        dx, dgl, dlam, dh0 = self.bwd(dh, x, gl, lam, h0, dh_last, c=c, threads=threads)
+        return dx, dgl, dlam, dh0, dz
 
 
 _default = None

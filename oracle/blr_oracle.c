@@ -173,6 +173,25 @@ void blr_oracle_bwd(int64_t B, int64_t L, int64_t D, double c, const double* dh,
   }
 }
 
+/* The merge that follows the BD-LRU in the gated recurrent layer (Alg. 1,
+ * H'_y = H_y (x) SiLU(H_z)): y = h * SiLU(z), SiLU(z) = z * sigmoid(z),
+ * elementwise over n values. */
+void blr_oracle_merge(int64_t n, const double* h, const double* z, double* y) {
+  for (int64_t k = 0; k < n; ++k) y[k] = h[k] * (z[k] * sigmoid(z[k]));
+}
+
+/* Backward of blr_oracle_merge for the upstream gradient dy (chain rule):
+ *   dh = dy * SiLU(z)
+ *   dz = dy * h * SiLU'(z),  SiLU'(z) = sigmoid(z) * (1 + z * (1 - sigmoid(z))). */
+void blr_oracle_merge_bwd(int64_t n, const double* dy, const double* h, const double* z,
+                          double* dh, double* dz) {
+  for (int64_t k = 0; k < n; ++k) {
+    const double sg = sigmoid(z[k]);
+    dh[k] = dy[k] * (z[k] * sg);
+    dz[k] = dy[k] * h[k] * (sg * (1.0 + z[k] * (1.0 - sg)));
+  }
+}
+
 /* One recurrent-inference step (low-cost inference, Sec. 1 and Sec. 4.3):
  * h_t = alpha_t h_prev + beta_t x_t for a batch of B states of width D.
  * x is (B, D), gl is (B, 2D). */

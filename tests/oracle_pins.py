@@ -14,7 +14,11 @@ the oracle disagrees with something the paper or mathematics fixes:
   * split / resume of the state;
   * the stability bound implied by alpha, beta in [0, 1] (Sec. 3.2);
   * central finite differences of every gradient, linearity of the gradient in
-    dh, and consistency of the single step with a length-1 scan.
+    dh, and consistency of the single step with a length-1 scan;
+  * for the merge of the gated layer (Alg. 1, y = h SiLU(z)): SiLU's values and
+    slope at 0 and its limits z -> +-inf, the reduction to the plain scan at
+    the z where SiLU(z) = 1 (found by root finding on scipy's expit), and
+    central finite differences of every gradient through the merge.
 
 They are plain functions (not tests) so that ``test_oracle_mutants.py`` can run
 the same set against oracle builds with a planted mistake and show that each
@@ -334,6 +338,80 @@ def pin_step(orc):
     assert _rel(ht, 0.5 * h_prev + math.sqrt(3) / 4 * x[:, 0]) < 1e-15
 
 
+# ----------------------------------------------------- the gated layer's merge
+
+
+def pin_merge_limits(orc):
+    rng = np.random.default_rng(23)
+    h = rng.standard_normal((3, 7, 4))
+    dy = rng.standard_normal(h.shape)
+    zeros = np.zeros_like(h)
+    # SiLU(0) = 0 and SiLU'(0) = 1/2
+    assert np.array_equal(orc.merge(h, zeros), zeros)
+    dh, dz = orc.merge_bwd(dy, h, zeros)
+    assert np.array_equal(dh, zeros)
+    assert _rel(dz, 0.5 * dy * h) < 1e-15
+    # z -> +inf: SiLU(z) / z -> 1 and SiLU'(z) -> 1; z -> -inf: both -> 0
+    big = np.full_like(h, 40.0)
+    assert _rel(orc.merge(h, big), 40.0 * h) < 1e-15
+    dh, dz = orc.merge_bwd(dy, h, big)
+    assert _rel(dh, 40.0 * dy) < 1e-15 and _rel(dz, dy * h) < 1e-15
+    y = orc.merge(h, -big)
+    assert np.max(np.abs(y)) <= 40.0 * math.exp(-40.0) * np.max(np.abs(h))
+    dh, dz = orc.merge_bwd(dy, h, -big)
+    assert np.max(np.abs(dz)) <= 41.0 * 40.0 * math.exp(-40.0) * np.max(np.abs(dy * h))
+
+
+def pin_merge_unit_gate(orc):
+    from scipy.optimize import brentq
+    z1 = brentq(lambda z: z * expit(z) - 1.0, 0.0, 5.0, xtol=1e-15, rtol=1e-15)  # SiLU(z1) = 1
+    rng = np.random.default_rng(24)
+    B, L, D, c = 2, 9, 3, 1.7
+    x, gl, lam = _rand_problem(rng, B, L, D)
+    h0 = rng.standard_normal((B, D))
+    dy = rng.standard_normal((B, L, D))
+    dh_last = rng.standard_normal((B, D))
+    z = np.full((B, L, D), z1)
+    y, yl = orc.fwd_gated(x, gl, lam, z, h0, c=c)
+    h, hl = orc.fwd(x, gl, lam, h0, c=c)
+    assert _rel(y, h) < 1e-14 and np.array_equal(yl, hl)
+    gated = orc.bwd_gated(dy, x, gl, lam, z, h0, dh_last, c=c)
+    plain = orc.bwd(dy, x, gl, lam, h0, dh_last, c=c)
+    for a, b in zip(gated[:4], plain):
+        assert _rel(a, b) < 1e-13
+
+
+def pin_gated_finite_differences(orc):
+    rng = np.random.default_rng(25)
+    B, L, D, c = 2, 5, 3, 0.8
+    x, gl, lam = _rand_problem(rng, B, L, D, decay=(0.6, 0.97))
+    z = 2.0 * rng.standard_normal((B, L, D))
+    h0 = rng.standard_normal((B, D))
+    dy = rng.standard_normal((B, L, D))
+    dh_last = rng.standard_normal((B, D))
+    dx, dgl, dlam, dh0, dz = orc.bwd_gated(dy, x, gl, lam, z, h0, dh_last, c=c)
+    eps = 1e-6
+
+    def loss(x_, gl_, lam_, z_, h0_):
+        y, yl = orc.fwd_gated(x_, gl_, lam_, z_, h0_, c=c)
+        return float(np.sum(dy * y) + np.sum(dh_last * yl))
+
+    def fd(arr, which):
+        out = np.empty_like(arr)
+        args = [x, gl, lam, z, h0]
+        for idx in np.ndindex(arr.shape):
+            p = arr.copy(); p[idx] += eps
+            m = arr.copy(); m[idx] -= eps
+            ap, am = list(args), list(args)
+            ap[which], am[which] = p, m
+            out[idx] = (loss(*ap) - loss(*am)) / (2 * eps)
+        return out
+
+    for got, arr, which, name in ((dx, x, 0, "dx"), (dgl, gl, 1, "dgl"), (dlam, lam, 2, "dlambda"),
+                                  (dz, z, 3, "dz"), (dh0, h0, 4, "dh0")):
+        assert _rel(got, fd(arr, which)) < 1e-6, name
+
+
 ALL_PINS = [
     pin_golden_forward,
     pin_geometric_closed_form,
@@ -349,4 +427,7 @@ ALL_PINS = [
     pin_finite_differences,
     pin_gradient_linearity,
     pin_step,
+    pin_merge_limits,
+    pin_merge_unit_gate,
+    pin_gated_finite_differences,
 ]

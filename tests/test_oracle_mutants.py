@@ -31,6 +31,9 @@ MUTANTS = [
      "gl[row * 2 * D + D + d], gl[row * 2 * D + d]", -1),
     ("h_{t-1} read one step late", "dx[row * D + d] = state; /* h_{t-1} */\n        gates_t gt = step_gates(c, s, gl[row * 2 * D + d], gl[row * 2 * D + D + d]);\n        state = gt.alpha * state + gt.beta * x[row * D + d];",
      "gates_t gt = step_gates(c, s, gl[row * 2 * D + d], gl[row * 2 * D + D + d]);\n        state = gt.alpha * state + gt.beta * x[row * D + d];\n        dx[row * D + d] = state;", 1),
+    ("merge gate without its z factor", "y[k] = h[k] * (z[k] * sigmoid(z[k]));", "y[k] = h[k] * sigmoid(z[k]);", 1),
+    ("merge slope without the z (1 - sigmoid) term", "(sg * (1.0 + z[k] * (1.0 - sg)))", "(sg * (1.0 + (1.0 - sg)))", 1),
+    ("merge passes dy through ungated", "dh[k] = dy[k] * (z[k] * sg);", "dh[k] = dy[k];", 1),
 ]
 
 
