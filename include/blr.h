@@ -147,6 +147,45 @@ BLR_API blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const floa
                         blr_stream_t stream);
 
 /*
+ * Forward scan fused with the merge of the gated recurrent layer (Alg. 1,
+ * H'_y = H_y (x) SiLU(H_z), the line after the BD-LRU):
+ *   y[b,t,d] = h[b,t,d] * SiLU(z[b,t,d]),   SiLU(z) = z * sigmoid(z),
+ * with h the scan of blr_scan_fwd, which is not written. Saves the separate
+ * merge's reading and writing of h.
+ * z           (B, L, D)  io dtype, the second branch's input (H_z)
+ * y           (B, L, D)  io dtype, output; may be NULL (then only h_last and
+ *                        the carries, as blr_scan_fwd with h == NULL)
+ * Other arguments, the workspace and the errors as blr_scan_fwd; z must be
+ * 16-byte aligned and no output may overlap an input. Problems of fewer than
+ * 256 chains (batch rows x groups of 32 float32 / 64 bfloat16 channels) run
+ * the scan and then an elementwise merge kernel over y in place.
+ */
+BLR_API blr_status blr_scan_fwd_gated(const blr_desc* desc, const void* x, const void* gate_logits,
+                                      const float* lambda, const float* h0, const void* z, void* y,
+                                      float* h_last, void* ws, size_t ws_bytes, blr_stream_t stream);
+
+/*
+ * Backward of blr_scan_fwd_gated for the loss
+ *   sum_{b,t,d} dy * y + sum_{b,d} dh_last * h_last:
+ * the scan's backward (outputs as blr_scan_bwd) for dh = dy * SiLU(z), and
+ *   dz = dy * h * SiLU'(z),   SiLU'(z) = sigmoid(z) (1 + z (1 - sigmoid(z))),
+ * with h recomputed, not read.
+ * dy          (B, L, D)  io dtype, upstream gradient of y
+ * z           (B, L, D)  io dtype, the forward's z
+ * dz          (B, L, D)  io dtype, output
+ * ws          the workspace of a blr_scan_fwd_gated (or blr_scan_fwd) of the same
+ *             desc and inputs, as for blr_scan_bwd.
+ * Other arguments as blr_scan_bwd; no output may overlap an input. Problems of
+ * fewer than 256 chains recompute h into dz, form dh in dx and dz in place with
+ * an elementwise kernel, then run the scan's backward from dx.
+ */
+BLR_API blr_status blr_scan_bwd_gated(const blr_desc* desc, const void* dy, const float* dh_last,
+                                      const void* x, const void* gate_logits, const float* lambda,
+                                      const float* h0, const void* z, void* dx, void* dgate_logits,
+                                      void* dz, float* dlambda, float* dh0, void* ws, size_t ws_bytes,
+                                      blr_stream_t stream);
+
+/*
  * One recurrent-inference step for a batch of states (the low-cost recurrent
  * inference of Sec. 1 and Sec. 4.3): h_t = alpha_t * h_prev + beta_t * x_t.
  * h_prev (B, D) float32; x_t (B, D) io dtype; gate_logits_t (B, 2D) io dtype;

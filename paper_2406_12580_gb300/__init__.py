@@ -13,6 +13,12 @@ there is no CPU path.
     blr_scan_bwd(desc, dh, dh_last, x, gate_logits, lam, h0, dx, dgate_logits, dlam, dh0, ws)
     blr_step(B, D, BLR_F32, 1.0, h_prev, x_t, gate_logits_t, lam, h_t)
 
+The gated recurrent layer's merge y = h SiLU(z) (Alg. 1) fused into the scan:
+
+    blr_scan_fwd_gated(desc, x, gate_logits, lam, h0, z, y, h_last, ws)
+    blr_scan_bwd_gated(desc, dy, dh_last, x, gate_logits, lam, h0, z, dx, dgate_logits, dz,
+                       dlam, dh0, ws)
+
 ``BDLRUScan`` wraps the forward and backward in a torch.autograd.Function.
 """
 from __future__ import annotations
@@ -25,7 +31,8 @@ from ._lib import (BLR_BF16, BLR_ERR_CUDA, BLR_ERR_INVALID_ARG, BLR_ERR_TIMEOUT,
 __all__ = [
     "BLR_F32", "BLR_BF16", "Desc", "BLRError", "blr_workspace_bytes", "blr_scan_fwd",
     "blr_scan_bwd", "blr_step", "blr_workspace_status", "blr_status_string",
-    "blr_selftest_wait_timeout", "blr_scan_fwd_noalloc", "BDLRUScan", "library_loaded",
+    "blr_selftest_wait_timeout", "blr_scan_fwd_noalloc", "blr_scan_fwd_gated", "blr_scan_bwd_gated",
+    "BDLRUScan", "library_loaded",
 ]
 
 
@@ -110,6 +117,28 @@ def blr_scan_bwd(desc, dh, dh_last, x, gate_logits, lam, h0, dx, dgate_logits, d
                                _ptr(dlam, "dlambda"), _ptr(dh0, "dh0"), _ptr(ws, "ws"), ws_bytes,
                                _stream(stream)),
            "blr_scan_bwd")
+
+
+def blr_scan_fwd_gated(desc, x, gate_logits, lam, h0, z, y, h_last, ws, stream=None):
+    ws_bytes = ws.numel() if ws is not None and not isinstance(ws, int) else blr_workspace_bytes(desc)
+    _check(load().blr_scan_fwd_gated(ctypes.byref(desc), _ptr(x, "x"),
+                                     _ptr(gate_logits, "gate_logits"), _ptr(lam, "lambda"),
+                                     _ptr(h0, "h0"), _ptr(z, "z"), _ptr(y, "y"),
+                                     _ptr(h_last, "h_last"), _ptr(ws, "ws"), ws_bytes,
+                                     _stream(stream)),
+           "blr_scan_fwd_gated")
+
+
+def blr_scan_bwd_gated(desc, dy, dh_last, x, gate_logits, lam, h0, z, dx, dgate_logits, dz, dlam,
+                       dh0, ws, stream=None):
+    ws_bytes = ws.numel() if ws is not None and not isinstance(ws, int) else blr_workspace_bytes(desc)
+    _check(load().blr_scan_bwd_gated(ctypes.byref(desc), _ptr(dy, "dy"), _ptr(dh_last, "dh_last"),
+                                     _ptr(x, "x"), _ptr(gate_logits, "gate_logits"),
+                                     _ptr(lam, "lambda"), _ptr(h0, "h0"), _ptr(z, "z"),
+                                     _ptr(dx, "dx"), _ptr(dgate_logits, "dgate_logits"),
+                                     _ptr(dz, "dz"), _ptr(dlam, "dlambda"), _ptr(dh0, "dh0"),
+                                     _ptr(ws, "ws"), ws_bytes, _stream(stream)),
+           "blr_scan_bwd_gated")
 
 
 def blr_step(B, D, io, c, h_prev, x_t, gate_logits_t, lam, h_t, stream=None):

@@ -12,6 +12,7 @@
 #include <cudaTypedefs.h>
 
 #include "blr.h"
+#include "blr_merge.cuh"
 #include "blr_seq.cuh"
 
 namespace {
@@ -231,21 +232,23 @@ blr_status allow_smem(K kernel, size_t smem) {
                     "set dynamic shared memory size");
 }
 
-template <typename T, class M, int VEC, int R, int RB>
+template <typename T, class M, int VEC, int R, int RB, bool GATED>
 blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB>;
-  a.stages = seq_stages(a.p.n_chain, 3 * (size_t)blr::seq_box_bytes<T, VEC, R>());
-  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, 3);
+  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED>;
+  constexpr int NB = GATED ? 4 : 3;
+  a.stages = seq_stages(a.p.n_chain, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
   BLR_TRY(allow_smem(kernel, smem));
   kernel<<<(unsigned)a.p.n_chain, 32, smem, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch seq_fwd_kernel");
 }
 
-template <typename T, class M, int VEC, int R, int RB>
+template <typename T, class M, int VEC, int R, int RB, bool GATED>
 blr_status launch_seq_bwd(blr::SeqBwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB>;
-  a.stages = seq_stages(a.p.n_chain, 4 * (size_t)blr::seq_box_bytes<T, VEC, R>());
-  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, 4);
+  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED>;
+  constexpr int NB = GATED ? 5 : 4;
+  a.stages = seq_stages(a.p.n_chain, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
   BLR_TRY(allow_smem(kernel, smem));
   kernel<<<(unsigned)a.p.n_chain, 32, smem, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch seq_bwd_kernel");
@@ -264,36 +267,57 @@ blr_status seq_maps_gl(CUtensorMap* mr, CUtensorMap* mi, const void* base, const
                          plan.D, plan.L, plan.B, rows, cols, 2 * plan.D);
 }
 
+// z given: the merge of the gated layer is fused, and h receives y = h SiLU(z).
 blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const float* lambda,
-                        const float* h0, void* h, float* h_last, unsigned char* w, cudaStream_t st) {
+                        const float* h0, void* h, float* h_last, unsigned char* w, cudaStream_t st,
+                        const void* z = nullptr) {
   blr::SeqFwdArgs a;
   BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.sr));
   BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, plan.sr));
   a.write_h = h != nullptr;
   if (a.write_h) BLR_TRY(seq_maps_x(&a.tm_h, h, plan, plan.sr));
   else memset(&a.tm_h, 0, sizeof(a.tm_h));
+  if (z != nullptr) BLR_TRY(seq_maps_x(&a.tm_z, z, plan, plan.sr));
+  else memset(&a.tm_z, 0, sizeof(a.tm_z));
   a.p = plan;
   a.lambda = lambda;
   a.h0 = h0;
   a.h_last = h_last;
   a.ws = w;
   a.stages = 2;
-  if (plan.io == BLR_F32) {
-    if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16>(a, st);
-    return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16>(a, st);
+  if (z != nullptr) {
+    if (plan.io == BLR_F32) {
+      if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, true>(a, st);
+      return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16, true>(a, st);
+    }
+    return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, true>(a, st);
   }
-  return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8>(a, st);
+  if (plan.io == BLR_F32) {
+    if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, false>(a, st);
+    return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16, false>(a, st);
+  }
+  return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, false>(a, st);
 }
 
+// z and dz given: dh is dy, the gradient of y = h SiLU(z), and dz is written.
 blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, const void* x,
                         const void* gl, const float* lambda, const float* h0, void* dx, void* dgl,
-                        float* dlambda, float* dh0, unsigned char* w, cudaStream_t st) {
+                        float* dlambda, float* dh0, unsigned char* w, cudaStream_t st,
+                        const void* z = nullptr, void* dz = nullptr) {
   blr::SeqBwdArgs a;
   BLR_TRY(seq_maps_x(&a.tm_dh, dh, plan, plan.srb));
   BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.srb));
   BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, plan.srb));
   BLR_TRY(seq_maps_x(&a.tm_dx, dx, plan, plan.srb));
   BLR_TRY(seq_maps_gl(&a.tm_dr, &a.tm_di, dgl, plan, plan.srb));
+  const bool gated = z != nullptr;
+  if (gated) {
+    BLR_TRY(seq_maps_x(&a.tm_z, z, plan, plan.srb));
+    BLR_TRY(seq_maps_x(&a.tm_dz, dz, plan, plan.srb));
+  } else {
+    memset(&a.tm_z, 0, sizeof(a.tm_z));
+    memset(&a.tm_dz, 0, sizeof(a.tm_dz));
+  }
   a.p = plan;
   a.dh_last = dh_last;
   a.lambda = lambda;
@@ -302,8 +326,12 @@ blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, 
   a.dh0 = dh0;
   a.ws = w;
   a.stages = 2;
-  if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16>(a, st);
-  return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8>(a, st);
+  if (gated) {
+    if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, true>(a, st);
+    return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, true>(a, st);
+  }
+  if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, false>(a, st);
+  return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false>(a, st);
 }
 
 // Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
@@ -323,44 +351,10 @@ blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fi
   return cuda_check(cudaGetLastError(), "launch prep_kernel");
 }
 
-}  // namespace
-
-extern "C" {
-
-size_t blr_workspace_bytes(const blr_desc* desc) {
-  Plan plan;
-  bool empty = false;
-  if (check_desc(desc, &plan, &empty) != BLR_OK || empty || desc->L == 0) return 0;
-  return plan.bytes;
-}
-
-blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_logits,
-                        const float* lambda, const float* h0, void* h, float* h_last, void* ws,
-                        size_t ws_bytes, blr_stream_t stream) {
-  Plan plan;
-  bool empty = false;
-  BLR_TRY(check_desc(desc, &plan, &empty));
-  if (empty) return BLR_OK;
-  BLR_TRY(need(lambda, "lambda", 16));
-  BLR_TRY(optional(h0, "h0", 4));
-  BLR_TRY(optional(h_last, "h_last", 4));
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const size_t state_bytes = sizeof(float) * (size_t)desc->B * (size_t)desc->D;
-  if (desc->L == 0) {  // empty sequence: the state is unchanged
-    if (h_last == nullptr) return BLR_OK;
-    if (h0 != nullptr)
-      return cuda_check(cudaMemcpyAsync(h_last, h0, state_bytes, cudaMemcpyDeviceToDevice, st),
-                        "copy h0 to h_last");
-    return cuda_check(cudaMemsetAsync(h_last, 0, state_bytes, st), "clear h_last");
-  }
-  BLR_TRY(need(x, "x", 16));
-  BLR_TRY(need(gate_logits, "gate_logits", 16));
-  BLR_TRY(optional(h, "h", 16));
-  BLR_TRY(check_ws(plan, ws, ws_bytes));
-
-  unsigned char* w = static_cast<unsigned char*>(ws);
-  if (plan.seq)  // serial kernels: no preparation
-    return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st);
+// The tiled look-back kernels: a preparation kernel, then the scan.
+blr_status scan_fwd_tiled(const Plan& plan, const blr_desc* desc, const void* x,
+                          const void* gate_logits, const float* lambda, const float* h0, void* h,
+                          float* h_last, unsigned char* w, cudaStream_t st) {
   // Clear the forward header (counters, error word), empty the
   // forward records, precompute k = -c softplus(Lambda).
   BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fpre,
@@ -380,51 +374,20 @@ blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_lo
     auto k = blr::scan_fwd_kernel<float, blr::MathPrecise>;
     const size_t smem = blr::ring_bytes<float, blr::fwd_stages<float>(), 3>();
     BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
-    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel"));
-  } else {
-    auto k = blr::scan_fwd_kernel<__nv_bfloat16, blr::MathFast>;
-    const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::fwd_stages<__nv_bfloat16>(), 3>();
-    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
-    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel"));
+    return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel");
   }
-  return BLR_OK;
+  auto k = blr::scan_fwd_kernel<__nv_bfloat16, blr::MathFast>;
+  const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::fwd_stages<__nv_bfloat16>(), 3>();
+  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
+  return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel");
 }
 
-blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
-                        const void* gate_logits, const float* lambda, const float* h0, void* dx,
-                        void* dgate_logits, float* dlambda, float* dh0, void* ws, size_t ws_bytes,
-                        blr_stream_t stream) {
-  Plan plan;
-  bool empty = false;
-  BLR_TRY(check_desc(desc, &plan, &empty));
-  if (empty) return BLR_OK;
-  BLR_TRY(need(lambda, "lambda", 16));
-  BLR_TRY(need(dlambda, "dlambda", 4));
-  BLR_TRY(optional(h0, "h0", 4));
-  BLR_TRY(optional(dh_last, "dh_last", 4));
-  BLR_TRY(optional(dh0, "dh0", 4));
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (desc->L == 0) {  // empty sequence: dh0 = dh_last, no dependence on Lambda
-    const size_t state_bytes = sizeof(float) * (size_t)desc->B * (size_t)desc->D;
-    BLR_TRY(cuda_check(cudaMemsetAsync(dlambda, 0, sizeof(float) * (size_t)desc->D, st),
-                       "clear dlambda"));
-    if (dh0 == nullptr) return BLR_OK;
-    if (dh_last != nullptr)
-      return cuda_check(cudaMemcpyAsync(dh0, dh_last, state_bytes, cudaMemcpyDeviceToDevice, st),
-                        "copy dh_last to dh0");
-    return cuda_check(cudaMemsetAsync(dh0, 0, state_bytes, st), "clear dh0");
-  }
-  BLR_TRY(need(dh, "dh", 16));
-  BLR_TRY(need(x, "x", 16));
-  BLR_TRY(need(gate_logits, "gate_logits", 16));
-  BLR_TRY(need(dx, "dx", 16));
-  BLR_TRY(need(dgate_logits, "dgate_logits", 16));
-  BLR_TRY(check_ws(plan, ws, ws_bytes));
-
-  unsigned char* w = static_cast<unsigned char*>(ws);
-  if (plan.seq)  // the forward cleared the counters and partial sums
-    return scan_bwd_seq(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
-                        dh0, w, st);
+// dh may be the dx buffer itself: every element of dh is read (into shared
+// memory, with its tile) before its tile writes dx.
+blr_status scan_bwd_tiled(const Plan& plan, const blr_desc* desc, const void* dh,
+                          const float* dh_last, const void* x, const void* gate_logits,
+                          const float* lambda, const float* h0, void* dx, void* dgate_logits,
+                          float* dlambda, float* dh0, unsigned char* w, cudaStream_t st) {
   // Clear the backward header and the dLambda partial sums, empty the backward
   // records (the forward's records stay: they hold the carries).
   BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, w + plan.off_bagg,
@@ -449,14 +412,180 @@ blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_la
     auto k = blr::scan_bwd_kernel<float, blr::MathPrecise>;
     const size_t smem = blr::ring_bytes<float, blr::bwd_stages<float>(), 4>();
     BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
-    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel"));
-  } else {
-    auto k = blr::scan_bwd_kernel<__nv_bfloat16, blr::MathFast>;
-    const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::bwd_stages<__nv_bfloat16>(), 4>();
-    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
-    BLR_TRY(launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel"));
+    return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel");
   }
-  return BLR_OK;
+  auto k = blr::scan_bwd_kernel<__nv_bfloat16, blr::MathFast>;
+  const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::bwd_stages<__nv_bfloat16>(), 4>();
+  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
+  return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel");
+}
+
+// Grid of the elementwise merge kernels: 16-byte vectors, 256 threads a block,
+// at most 8 blocks per SM (grid-stride beyond).
+unsigned merge_grid(int64_t n_vec) {
+  int64_t blocks = (n_vec + 255) / 256;
+  const int64_t cap = (int64_t)sm_count() * 8;
+  if (blocks > cap) blocks = cap;
+  return (unsigned)(blocks > 0 ? blocks : 1);
+}
+
+blr_status launch_merge_fwd(int io, void* y, const void* z, int64_t n, cudaStream_t st) {
+  if (io == BLR_F32) {
+    const int64_t nv = n / 4;
+    blr::merge_fwd_kernel<float><<<merge_grid(nv), 256, 0, st>>>(static_cast<float*>(y),
+                                                                 static_cast<const float*>(z), nv);
+  } else {
+    const int64_t nv = n / 8;
+    blr::merge_fwd_kernel<__nv_bfloat16><<<merge_grid(nv), 256, 0, st>>>(
+        static_cast<__nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(z), nv);
+  }
+  return cuda_check(cudaGetLastError(), "launch merge_fwd_kernel");
+}
+
+blr_status launch_merge_bwd(int io, const void* dy, const void* z, void* dh, void* hz, int64_t n,
+                            cudaStream_t st) {
+  if (io == BLR_F32) {
+    const int64_t nv = n / 4;
+    blr::merge_bwd_kernel<float><<<merge_grid(nv), 256, 0, st>>>(
+        static_cast<const float*>(dy), static_cast<const float*>(z), static_cast<float*>(dh),
+        static_cast<float*>(hz), nv);
+  } else {
+    const int64_t nv = n / 8;
+    using bf = __nv_bfloat16;
+    blr::merge_bwd_kernel<bf><<<merge_grid(nv), 256, 0, st>>>(
+        static_cast<const bf*>(dy), static_cast<const bf*>(z), static_cast<bf*>(dh),
+        static_cast<bf*>(hz), nv);
+  }
+  return cuda_check(cudaGetLastError(), "launch merge_bwd_kernel");
+}
+
+// blr_scan_fwd (z == NULL) and blr_scan_fwd_gated (z given; h is then y).
+blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_logits,
+                          const float* lambda, const float* h0, const void* z, void* h,
+                          float* h_last, void* ws, size_t ws_bytes, blr_stream_t stream,
+                          bool gated) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty) return BLR_OK;
+  BLR_TRY(need(lambda, "lambda", 16));
+  BLR_TRY(optional(h0, "h0", 4));
+  BLR_TRY(optional(h_last, "h_last", 4));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const size_t state_bytes = sizeof(float) * (size_t)desc->B * (size_t)desc->D;
+  if (desc->L == 0) {  // empty sequence: the state is unchanged
+    if (h_last == nullptr) return BLR_OK;
+    if (h0 != nullptr)
+      return cuda_check(cudaMemcpyAsync(h_last, h0, state_bytes, cudaMemcpyDeviceToDevice, st),
+                        "copy h0 to h_last");
+    return cuda_check(cudaMemsetAsync(h_last, 0, state_bytes, st), "clear h_last");
+  }
+  BLR_TRY(need(x, "x", 16));
+  BLR_TRY(need(gate_logits, "gate_logits", 16));
+  BLR_TRY(optional(h, gated ? "y" : "h", 16));
+  if (gated) BLR_TRY(need(z, "z", 16));
+  BLR_TRY(check_ws(plan, ws, ws_bytes));
+
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  if (plan.seq)  // serial kernels (the merge fused): no preparation
+    return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st, h != nullptr ? z : nullptr);
+  BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, h, h_last, w, st));
+  if (z == nullptr || h == nullptr) return BLR_OK;
+  return launch_merge_fwd(desc->io, h, z, desc->B * desc->L * desc->D, st);
+}
+
+// blr_scan_bwd (z == NULL; dh is the gradient of h) and blr_scan_bwd_gated
+// (z and dz given; dh is the gradient dy of y = h SiLU(z)).
+blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
+                          const void* gate_logits, const float* lambda, const float* h0,
+                          const void* z, void* dx, void* dgate_logits, void* dz, float* dlambda,
+                          float* dh0, void* ws, size_t ws_bytes, blr_stream_t stream, bool gated) {
+  Plan plan;
+  bool empty = false;
+  BLR_TRY(check_desc(desc, &plan, &empty));
+  if (empty) return BLR_OK;
+  BLR_TRY(need(lambda, "lambda", 16));
+  BLR_TRY(need(dlambda, "dlambda", 4));
+  BLR_TRY(optional(h0, "h0", 4));
+  BLR_TRY(optional(dh_last, "dh_last", 4));
+  BLR_TRY(optional(dh0, "dh0", 4));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (desc->L == 0) {  // empty sequence: dh0 = dh_last, no dependence on Lambda
+    const size_t state_bytes = sizeof(float) * (size_t)desc->B * (size_t)desc->D;
+    BLR_TRY(cuda_check(cudaMemsetAsync(dlambda, 0, sizeof(float) * (size_t)desc->D, st),
+                       "clear dlambda"));
+    if (dh0 == nullptr) return BLR_OK;
+    if (dh_last != nullptr)
+      return cuda_check(cudaMemcpyAsync(dh0, dh_last, state_bytes, cudaMemcpyDeviceToDevice, st),
+                        "copy dh_last to dh0");
+    return cuda_check(cudaMemsetAsync(dh0, 0, state_bytes, st), "clear dh0");
+  }
+  BLR_TRY(need(dh, gated ? "dy" : "dh", 16));
+  if (gated) {
+    BLR_TRY(need(z, "z", 16));
+    BLR_TRY(need(dz, "dz", 16));
+  }
+  BLR_TRY(need(x, "x", 16));
+  BLR_TRY(need(gate_logits, "gate_logits", 16));
+  BLR_TRY(need(dx, "dx", 16));
+  BLR_TRY(need(dgate_logits, "dgate_logits", 16));
+  BLR_TRY(check_ws(plan, ws, ws_bytes));
+
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  if (plan.seq)  // the forward cleared the counters and partial sums
+    return scan_bwd_seq(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
+                        dh0, w, st, z, dz);
+  if (z == nullptr)
+    return scan_bwd_tiled(plan, desc, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
+                          dlambda, dh0, w, st);
+  // Gated, tiled: h recomputed into dz (a forward of the same problem, which
+  // also rewrites the same carries), then dh = dy SiLU(z) into dx and
+  // dz = dy h SiLU'(z), then the scan's backward from dh in dx.
+  BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, dz, nullptr, w, st));
+  BLR_TRY(launch_merge_bwd(desc->io, dh, z, dx, dz, desc->B * desc->L * desc->D, st));
+  return scan_bwd_tiled(plan, desc, dx, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
+                        dlambda, dh0, w, st);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t blr_workspace_bytes(const blr_desc* desc) {
+  Plan plan;
+  bool empty = false;
+  if (check_desc(desc, &plan, &empty) != BLR_OK || empty || desc->L == 0) return 0;
+  return plan.bytes;
+}
+
+blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_logits,
+                        const float* lambda, const float* h0, void* h, float* h_last, void* ws,
+                        size_t ws_bytes, blr_stream_t stream) {
+  return scan_fwd_entry(desc, x, gate_logits, lambda, h0, nullptr, h, h_last, ws, ws_bytes, stream,
+                        false);
+}
+
+blr_status blr_scan_fwd_gated(const blr_desc* desc, const void* x, const void* gate_logits,
+                              const float* lambda, const float* h0, const void* z, void* y,
+                              float* h_last, void* ws, size_t ws_bytes, blr_stream_t stream) {
+  return scan_fwd_entry(desc, x, gate_logits, lambda, h0, z, y, h_last, ws, ws_bytes, stream, true);
+}
+
+blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
+                        const void* gate_logits, const float* lambda, const float* h0, void* dx,
+                        void* dgate_logits, float* dlambda, float* dh0, void* ws, size_t ws_bytes,
+                        blr_stream_t stream) {
+  return scan_bwd_entry(desc, dh, dh_last, x, gate_logits, lambda, h0, nullptr, dx, dgate_logits,
+                        nullptr, dlambda, dh0, ws, ws_bytes, stream, false);
+}
+
+blr_status blr_scan_bwd_gated(const blr_desc* desc, const void* dy, const float* dh_last,
+                              const void* x, const void* gate_logits, const float* lambda,
+                              const float* h0, const void* z, void* dx, void* dgate_logits,
+                              void* dz, float* dlambda, float* dh0, void* ws, size_t ws_bytes,
+                              blr_stream_t stream) {
+  return scan_bwd_entry(desc, dy, dh_last, x, gate_logits, lambda, h0, z, dx, dgate_logits, dz,
+                        dlambda, dh0, ws, ws_bytes, stream, true);
 }
 
 blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_prev,

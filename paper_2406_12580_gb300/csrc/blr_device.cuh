@@ -271,11 +271,20 @@ __device__ __forceinline__ float expm1_neg(float l) {
   return l > -kExpm1Series ? e : ex2_approx(l * 1.4426950408889634f) - 1.0f;
 }
 
+// SiLU(z) = z sigmoid(z) and SiLU'(z) = sigmoid(z) (1 + z (1 - sigmoid(z))), the
+// merge gate of the gated recurrent layer (Alg. 1), on the value as the policy
+// unpacks it (z itself for GatesPrecise, z/2 for GatesFast).
 struct GatesPrecise : MathPrecise {
   static constexpr int kDeg = 6;
   static constexpr bool kHalfInputs = false;
   static __device__ __forceinline__ float decay_log(float rho, float k, float) {
     return k * sigmoid(rho);
+  }
+  static __device__ __forceinline__ float silu(float z) { return z * sigmoid(z); }
+  static __device__ __forceinline__ void silu_grad(float z, float& f, float& df) {
+    const float sg = sigmoid(z);
+    f = z * sg;
+    df = fmaf(sg, z - f, sg);  // z (1 - sg) = z - f
   }
 };
 
@@ -295,6 +304,15 @@ struct GatesFast : MathFast {
   }
   static __device__ __forceinline__ float decay_log(float rho, float, float kh) {
     return fmaf(kh, tanh_approx(0.5f * rho), kh);
+  }
+  // With hz = z/2 and th = tanh(hz): SiLU = hz (1 + th), sigmoid = (1 + th)/2
+  // and z (1 - sigmoid) = hz (1 - th).
+  static __device__ __forceinline__ float silu(float hz) { return fmaf(hz, tanh_approx(hz), hz); }
+  static __device__ __forceinline__ void silu_grad(float hz, float& f, float& df) {
+    const float th = tanh_approx(hz);
+    const float sg = fmaf(0.5f, th, 0.5f);
+    f = fmaf(hz, th, hz);
+    df = fmaf(sg, fmaf(-hz, th, hz), sg);
   }
 };
 

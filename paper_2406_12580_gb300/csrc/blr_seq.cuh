@@ -41,7 +41,8 @@ struct SeqFwdArgs {
   CUtensorMap tm_x;
   CUtensorMap tm_r;
   CUtensorMap tm_i;
-  CUtensorMap tm_h;  // unused when h is NULL
+  CUtensorMap tm_h;  // h, or y = h SiLU(z) when gated; unused when NULL
+  CUtensorMap tm_z;  // gated: z, the merge gate's input
   Plan p;
   const float* lambda;
   const float* h0;
@@ -59,6 +60,8 @@ struct SeqBwdArgs {
   CUtensorMap tm_dx;
   CUtensorMap tm_dr;
   CUtensorMap tm_di;
+  CUtensorMap tm_z;   // gated: z
+  CUtensorMap tm_dz;  // gated: dz
   Plan p;
   const float* dh_last;
   const float* lambda;
@@ -114,8 +117,10 @@ struct SeqRing {
 
 // One stage, rows [0, rows) (all R when FULL). Phase 1 evaluates the
 // gates of every row (independent work), phase 2 runs the recurrence and
-// writes h over x in the stage. `cidx` is the index of the next kept state.
-template <class IO, class G, bool POLY, bool FULL, int R, int RB>
+// writes h over x in the stage (GATED: y = h SiLU(z), the merge of the gated
+// recurrent layer, Alg. 1, with z the stage's fourth box). `cidx` is the index
+// of the next kept state.
+template <class IO, class G, bool POLY, bool FULL, int R, int RB, bool GATED>
 __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
                                               const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
                                               float (&hc)[IO::VEC], float* carry, int64_t& cidx,
@@ -124,11 +129,20 @@ __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
   constexpr int V = IO::VEC;
   constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
   constexpr uint32_t BOX = R * ROWB;
-  float al[R][V], uu[R][V];
+  float al[R][V], uu[R][V], sz[GATED ? R : 1][V];
 #pragma unroll
   for (int s = 0; s < R; ++s) {
     if (FULL || s < rows) {
       float xv[V], rv[V], iv[V];
+      if constexpr (GATED) {
+        float zv[V];
+        if constexpr (G::kHalfInputs)
+          IO::unpack_half(*reinterpret_cast<const Raw*>(sb + 3 * BOX + s * ROWB), zv);
+        else
+          IO::unpack(*reinterpret_cast<const Raw*>(sb + 3 * BOX + s * ROWB), zv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) sz[s][v] = G::silu(zv[v]);
+      }
       if constexpr (G::kHalfInputs) {
         IO::unpack_half(*reinterpret_cast<const Raw*>(sb + s * ROWB), xv);
         IO::unpack_half(*reinterpret_cast<const Raw*>(sb + BOX + s * ROWB), rv);
@@ -159,7 +173,10 @@ __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
 #pragma unroll
       for (int v = 0; v < V; ++v) {
         hc[v] = fmaf(al[s][v], hc[v], uu[s][v]);
-        out[v] = hc[v];
+        if constexpr (GATED)
+          out[v] = hc[v] * sz[s][v];
+        else
+          out[v] = hc[v];
       }
       IO::store_smem(sb + s * ROWB, out);
       if ((s + 1) % RB == 0) {  // a kept state: after step (cidx + 1) RB - 1
@@ -173,16 +190,17 @@ __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
   }
 }
 
-template <typename T, class M, int VEC, int R, int RB>
+template <typename T, class M, int VEC, int R, int RB, bool GATED>
 __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ SeqFwdArgs a) {
   using IO = Io<T, VEC>;
   using G = typename GatePolicy<M>::type;
   constexpr int CHW = 32 * VEC;
+  constexpr int NB = GATED ? 4 : 3;  // boxes per stage: x, rho, iota (, z)
   constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
   static_assert(R % RB == 0, "kept states must fall on stage rows");
   const Plan& p = a.p;
   extern __shared__ unsigned char seq_smem[];
-  SeqRing<3, BOX> ring{align128(seq_smem), nullptr, a.stages};
+  SeqRing<NB, BOX> ring{align128(seq_smem), nullptr, a.stages};
   ring.bars = reinterpret_cast<uint64_t*>(ring.stage(ring.S));
 
   const int lane = threadIdx.x;
@@ -216,10 +234,11 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
   auto issue = [&](int st, int64_t j) {
     unsigned char* dst = ring.stage(st);
     const int t = (int)(j * R);
-    mbar_arrive_expect_tx(&ring.bars[st], 3 * BOX);
+    mbar_arrive_expect_tx(&ring.bars[st], NB * BOX);
     tma_load_3d(dst, &a.tm_x, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + BOX, &a.tm_r, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + 2 * BOX, &a.tm_i, &ring.bars[st], cd, t, cb);
+    if constexpr (GATED) tma_load_3d(dst + 3 * BOX, &a.tm_z, &ring.bars[st], cd, t, cb);
   };
   if (lane == 0) {
     for (int s = 0; s < ring.S; ++s) mbar_init(&ring.bars[s], 1);
@@ -246,11 +265,11 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     const int rows = (int)(left < R ? left : R);
     if (rows == R) {
       if (poly)
-        seq_fwd_stage<IO, G, true, true, R, RB>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
+        seq_fwd_stage<IO, G, true, true, R, RB, GATED>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
       else
-        seq_fwd_stage<IO, G, false, true, R, RB>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
+        seq_fwd_stage<IO, G, false, true, R, RB, GATED>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
     } else {
-      seq_fwd_stage<IO, G, false, false, R, RB>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
+      seq_fwd_stage<IO, G, false, false, R, RB, GATED>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
     }
     fence_proxy_async_smem();  // the stage's h rows, visible to the TMA store
     __syncwarp();
@@ -276,8 +295,10 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
 // One sub-block of RB steps (rows [0, srows) when not FULL) starting at row
 // `row0` of the stage: forward recompute from the state hc, then the reverse
 // recurrence carrying w = alpha g. dx, d rho and d iota overwrite dh, rho and
-// iota of the same rows in the stage.
-template <class IO, class G, bool POLY, bool FULL, int R, int RB>
+// iota of the same rows in the stage. GATED: the first box holds dy, the
+// gradient of y = h SiLU(z) (Alg. 1), so dh = dy SiLU(z), and
+// dz = dy h SiLU'(z) overwrites z in the fifth box.
+template <class IO, class G, bool POLY, bool FULL, int R, int RB, bool GATED>
 __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int srows,
                                             const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
                                             float (&hc)[IO::VEC], float (&w)[IO::VEC],
@@ -286,11 +307,12 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
   constexpr int V = IO::VEC;
   constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
   constexpr uint32_t BOX = R * ROWB;
-  // boxes of a backward stage: dh, x, rho, iota
+  // boxes of a backward stage: dh (dy), x, rho, iota (, z)
   unsigned char* s_dh = lb + row0 * ROWB;
   const unsigned char* s_x = s_dh + BOX;
   unsigned char* s_r = s_dh + 2 * BOX;
   unsigned char* s_i = s_dh + 3 * BOX;
+  unsigned char* s_z = s_dh + 4 * BOX;
   float E[RB][V], RS[RB][V], HP[RB][V];
 #pragma unroll
   for (int s = 0; s < RB; ++s) {
@@ -330,8 +352,17 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
 #pragma unroll
   for (int s = RB - 1; s >= 0; --s) {
     if (FULL || s < srows) {
-      float gv[V], xv[V], rv[V], iv[V], ox[V], orho[V], oiota[V];
+      float gv[V], xv[V], rv[V], iv[V], ox[V], orho[V], oiota[V], sf[V], sdf[V], oz[V];
       IO::unpack(*reinterpret_cast<const Raw*>(s_dh + s * ROWB), gv);
+      if constexpr (GATED) {
+        float zv[V];
+        if constexpr (G::kHalfInputs)
+          IO::unpack_half(*reinterpret_cast<const Raw*>(s_z + s * ROWB), zv);
+        else
+          IO::unpack(*reinterpret_cast<const Raw*>(s_z + s * ROWB), zv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) G::silu_grad(zv[v], sf[v], sdf[v]);
+      }
       IO::unpack(*reinterpret_cast<const Raw*>(s_x + s * ROWB), xv);
       if constexpr (G::kHalfInputs) {
         IO::unpack_half(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
@@ -353,10 +384,13 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
           r = G::sigmoid(rv[v]);
           i = G::sigmoid(iv[v]);
         }
-        const float g = gv[v] + w[v];
+        float dhv = gv[v];
+        if constexpr (GATED) dhv *= sf[v];
+        const float g = dhv + w[v];
         w[v] = alpha * g;
         const float ix = i * xv[v];
         const float u = (q * rs) * ix;
+        if constexpr (GATED) oz[v] = (gv[v] * fmaf(alpha, HP[s][v], u)) * sdf[v];  // dy h_t SiLU'
         ox[v] = (g * (q * rs)) * i;
         oiota[v] = (g * u) * (1.0f - i);
         // d/dl of h_t: alpha g (h_{t-1} - alpha u / q), with alpha g = w and
@@ -368,21 +402,23 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
       IO::store_smem(s_dh + s * ROWB, ox);
       IO::store_smem(s_r + s * ROWB, orho);
       IO::store_smem(s_i + s * ROWB, oiota);
+      if constexpr (GATED) IO::store_smem(s_z + s * ROWB, oz);
     }
   }
 }
 
-template <typename T, class M, int VEC, int R, int RB>
+template <typename T, class M, int VEC, int R, int RB, bool GATED>
 __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(const __grid_constant__ SeqBwdArgs a) {
   using IO = Io<T, VEC>;
   using G = typename GatePolicy<M>::type;
   constexpr int CHW = 32 * VEC;
+  constexpr int NB = GATED ? 5 : 4;  // boxes per stage: dh (dy), x, rho, iota (, z)
   constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
   constexpr int NSUB = R / RB;
   static_assert(R % RB == 0, "sub-blocks must tile a stage");
   const Plan& p = a.p;
   extern __shared__ unsigned char seq_smem[];
-  SeqRing<4, BOX> ring{align128(seq_smem), nullptr, a.stages};
+  SeqRing<NB, BOX> ring{align128(seq_smem), nullptr, a.stages};
   ring.bars = reinterpret_cast<uint64_t*>(ring.stage(ring.S));
 
   const int lane = threadIdx.x;
@@ -433,11 +469,12 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   auto issue = [&](int st, int64_t j) {
     unsigned char* dst = ring.stage(st);
     const int t = (int)(j * R);
-    mbar_arrive_expect_tx(&ring.bars[st], 4 * BOX);
+    mbar_arrive_expect_tx(&ring.bars[st], NB * BOX);
     tma_load_3d(dst, &a.tm_dh, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + BOX, &a.tm_x, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + 2 * BOX, &a.tm_r, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + 3 * BOX, &a.tm_i, &ring.bars[st], cd, t, cb);
+    if constexpr (GATED) tma_load_3d(dst + 4 * BOX, &a.tm_z, &ring.bars[st], cd, t, cb);
   };
   if (lane == 0) {
     for (int s = 0; s < ring.S; ++s) mbar_init(&ring.bars[s], 1);
@@ -483,11 +520,11 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
         if (m - QD >= 0) load_start(m - QD, sq[QD - 1]);  // in flight for QD sub-blocks
         if (srows == RB) {
           if (poly)
-            seq_bwd_sub<IO, G, true, true, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
+            seq_bwd_sub<IO, G, true, true, R, RB, GATED>(lb, row0, srows, k, kh, hc, w, dlr);
           else
-            seq_bwd_sub<IO, G, false, true, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
+            seq_bwd_sub<IO, G, false, true, R, RB, GATED>(lb, row0, srows, k, kh, hc, w, dlr);
         } else {
-          seq_bwd_sub<IO, G, false, false, R, RB>(lb, row0, srows, k, kh, hc, w, dlr);
+          seq_bwd_sub<IO, G, false, false, R, RB, GATED>(lb, row0, srows, k, kh, hc, w, dlr);
         }
         --m;
       }
@@ -499,6 +536,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
       tma_store_3d(&a.tm_dx, sb, cd, t, cb);
       tma_store_3d(&a.tm_dr, sb + 2 * BOX, cd, t, cb);
       tma_store_3d(&a.tm_di, sb + 3 * BOX, cd, t, cb);
+      if constexpr (GATED) tma_store_3d(&a.tm_dz, sb + 4 * BOX, cd, t, cb);
       bulk_commit();
     }
     prev = st;

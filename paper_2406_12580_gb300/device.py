@@ -11,8 +11,8 @@ from typing import Optional
 
 import numpy as np
 
-from . import (BLR_BF16, BLR_F32, Desc, blr_scan_bwd, blr_scan_fwd, blr_step,
-               blr_workspace_bytes)
+from . import (BLR_BF16, BLR_F32, Desc, blr_scan_bwd, blr_scan_bwd_gated, blr_scan_fwd,
+               blr_scan_fwd_gated, blr_step, blr_workspace_bytes)
 from .inputs import BF16, ScanInputs, StepInputs
 
 
@@ -61,6 +61,8 @@ class ScanBuffers:
     dlam: object
     dh0: object
     ws: object
+    z: object = None   # gated workloads: the merge's input (then h holds y and dh is dy)
+    dz: object = None
 
     @classmethod
     def from_inputs(cls, inp: ScanInputs, device="cuda", with_bwd: bool = True):
@@ -84,7 +86,9 @@ class ScanBuffers:
         dgl = torch.empty(B, L, 2 * D, dtype=io_t, device=device) if bwd else None
         dlam = torch.empty(D, dtype=f32, device=device) if bwd else None
         dh0 = torch.empty(B, D, dtype=f32, device=device) if bwd else None
-        return cls(desc, x, gl, lam, h0, dh, dh_last, h, h_last, dx, dgl, dlam, dh0, ws)
+        z = up("z") if inp.z is not None else None
+        dz = torch.empty(B, L, D, dtype=io_t, device=device) if (bwd and z is not None) else None
+        return cls(desc, x, gl, lam, h0, dh, dh_last, h, h_last, dx, dgl, dlam, dh0, ws, z, dz)
 
     def fwd(self, stream=None, write_h: bool = True):
         blr_scan_fwd(self.desc, self.x, self.gl, self.lam, self.h0, self.h if write_h else None,
@@ -93,6 +97,16 @@ class ScanBuffers:
     def bwd(self, stream=None):
         blr_scan_bwd(self.desc, self.dh, self.dh_last, self.x, self.gl, self.lam, self.h0, self.dx,
                      self.dgl, self.dlam, self.dh0, self.ws, stream)
+
+    def fwd_gated(self, stream=None):
+        """y = h SiLU(z) into self.h."""
+        blr_scan_fwd_gated(self.desc, self.x, self.gl, self.lam, self.h0, self.z, self.h,
+                           self.h_last, self.ws, stream)
+
+    def bwd_gated(self, stream=None):
+        """Backward of fwd_gated with self.dh as dy."""
+        blr_scan_bwd_gated(self.desc, self.dh, self.dh_last, self.x, self.gl, self.lam, self.h0,
+                           self.z, self.dx, self.dgl, self.dz, self.dlam, self.dh0, self.ws, stream)
 
 
 @dataclass

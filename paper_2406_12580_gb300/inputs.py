@@ -65,6 +65,7 @@ class ScanConfig:
     random_h0: bool = False
     random_dh_last: bool = False
     c: float = 1.0
+    gated: bool = False                # also draw z, the gated layer's merge input (Alg. 1)
 
     @property
     def elements(self) -> int:
@@ -119,6 +120,7 @@ class ScanInputs:
     h0: Optional[np.ndarray]   # (B, D) float32 or None (zero state)
     dh_last: Optional[np.ndarray]  # (B, D) float32 or None
     bits: dict = field(default_factory=dict)
+    z: Optional[np.ndarray] = None     # (B, L, D) float32 when cfg.gated (dh is then dy)
 
     def io_array(self, name: str) -> np.ndarray:
         """The array as the device sees it: float32, or uint16 bf16 bits."""
@@ -176,6 +178,9 @@ def make_scan_inputs(cfg: ScanConfig) -> ScanInputs:
     del gl
     if dh is not None:
         inp.dh, bits["dh"] = _to_io(dh, cfg.io)
+    if cfg.gated:  # a stream of its own, so the other arrays do not depend on it
+        z = _normal(np.random.default_rng([cfg.seed, 2]), n, 1.0).reshape(B, L, D)
+        inp.z, bits["z"] = _to_io(z, cfg.io)
     inp.bits = {k: v for k, v in bits.items() if v is not None}
     return inp
 

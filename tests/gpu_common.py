@@ -38,6 +38,17 @@ def gpu_scan(inp: I.ScanInputs, with_bwd=True, sync=True):
     return buf
 
 
+def gpu_scan_gated(inp: I.ScanInputs, with_bwd=True):
+    """The gated entry points (y = h SiLU(z) in buf.h; dz in buf.dz)."""
+    import torch
+    buf = ScanBuffers.from_inputs(inp, with_bwd=with_bwd)
+    buf.fwd_gated()
+    if with_bwd and buf.dh is not None:
+        buf.bwd_gated()
+    torch.cuda.synchronize()
+    return buf
+
+
 def gpu_outputs(buf, dsel=None):
     """Outputs as float64 numpy arrays, optionally only the channels `dsel`."""
     import torch
@@ -61,6 +72,8 @@ def gpu_outputs(buf, dsel=None):
         out["dgl"] = take(buf.dgl, 2 * D)
         out["dlam"] = take(buf.dlam, D)
         out["dh0"] = take(buf.dh0, D)
+    if buf.dz is not None:
+        out["dz"] = take(buf.dz, D)
     return out
 
 
@@ -71,16 +84,27 @@ def select_channels(inp: I.ScanInputs, dsel):
     gidx = np.concatenate([dsel, dsel + D])
     pick = lambda a, ax_idx: None if a is None else np.ascontiguousarray(a[..., ax_idx])  # noqa: E731
     return dict(x=pick(inp.x, dsel), gl=pick(inp.gl, gidx), lam=inp.lam[dsel],
-                h0=pick(inp.h0, dsel), dh=pick(inp.dh, dsel), dh_last=pick(inp.dh_last, dsel))
+                h0=pick(inp.h0, dsel), dh=pick(inp.dh, dsel), dh_last=pick(inp.dh_last, dsel),
+                z=pick(inp.z, dsel))
 
 
 def oracle_outputs(inp: I.ScanInputs, dsel=None, threads=0):
     orc = oracle.load()
     cfg = inp.cfg
     if dsel is None:
-        a = dict(x=inp.x, gl=inp.gl, lam=inp.lam, h0=inp.h0, dh=inp.dh, dh_last=inp.dh_last)
+        a = dict(x=inp.x, gl=inp.gl, lam=inp.lam, h0=inp.h0, dh=inp.dh, dh_last=inp.dh_last,
+                 z=inp.z)
     else:
         a = select_channels(inp, dsel)
+    if a["z"] is not None:  # the gated layer: h holds y = h SiLU(z), dh is dy
+        y, h_last = orc.fwd_gated(a["x"], a["gl"], a["lam"], a["z"], a["h0"], c=cfg.c,
+                                  threads=threads)
+        out = {"h": y, "h_last": h_last}
+        if a["dh"] is not None:
+            dx, dgl, dlam, dh0, dz = orc.bwd_gated(a["dh"], a["x"], a["gl"], a["lam"], a["z"],
+                                                   a["h0"], a["dh_last"], c=cfg.c, threads=threads)
+            out.update(dx=dx, dgl=dgl, dlam=dlam, dh0=dh0, dz=dz)
+        return out
     h, h_last = orc.fwd(a["x"], a["gl"], a["lam"], a["h0"], c=cfg.c, threads=threads)
     out = {"h": h, "h_last": h_last}
     if a["dh"] is not None:

@@ -116,6 +116,33 @@ def test_bwd_validation(lib):
                ws=None) == _lib.BLR_OK
 
 
+def fwd_gated(lib, desc, z=FAKE, y=FAKE):
+    ws_bytes = lib.blr_workspace_bytes(ctypes.byref(desc))
+    return lib.blr_scan_fwd_gated(ctypes.byref(desc), FAKE, FAKE, FAKE, None, z, y, None, FAKE,
+                                  ws_bytes, None)
+
+
+def bwd_gated(lib, desc, z=FAKE, dz=FAKE, dy=FAKE):
+    ws_bytes = lib.blr_workspace_bytes(ctypes.byref(desc))
+    return lib.blr_scan_bwd_gated(ctypes.byref(desc), dy, None, FAKE, FAKE, FAKE, None, z, FAKE,
+                                  FAKE, dz, FAKE, None, FAKE, ws_bytes, None)
+
+
+def test_gated_validation(lib):
+    assert fwd_gated(lib, D(2, 4, 8), z=None) == _lib.BLR_ERR_INVALID_ARG
+    assert b"z is NULL" in lib.blr_last_error_string()
+    assert fwd_gated(lib, D(2, 4, 8), z=FAKE + 8) == _lib.BLR_ERR_INVALID_ARG
+    assert fwd_gated(lib, D(2, 4, 8), y=FAKE + 2) == _lib.BLR_ERR_INVALID_ARG
+    assert fwd_gated(lib, D(2, 4, 12), z=None) == _lib.BLR_ERR_UNSUPPORTED  # the shape first
+    assert fwd_gated(lib, D(0, 4, 8), z=None, y=None) == _lib.BLR_OK
+    assert bwd_gated(lib, D(2, 4, 8), z=None) == _lib.BLR_ERR_INVALID_ARG
+    assert bwd_gated(lib, D(2, 4, 8), dz=None) == _lib.BLR_ERR_INVALID_ARG
+    assert b"dz is NULL" in lib.blr_last_error_string()
+    assert bwd_gated(lib, D(2, 4, 8), dz=FAKE + 4) == _lib.BLR_ERR_INVALID_ARG
+    assert bwd_gated(lib, D(2, 4, 8), dy=None) == _lib.BLR_ERR_INVALID_ARG
+    assert b"dy is NULL" in lib.blr_last_error_string()
+
+
 def test_step_validation(lib):
     f = lib.blr_step
     assert f(-1, 8, 0, 1.0, FAKE, FAKE, FAKE, FAKE, FAKE, None) == _lib.BLR_ERR_INVALID_ARG

@@ -8,7 +8,8 @@ bfloat16 I/O.
 import numpy as np
 import pytest
 
-from gpu_common import (TOL, compare, gpu_outputs, gpu_scan, gpu_step, normwise, oracle_outputs)
+from gpu_common import (TOL, compare, gpu_outputs, gpu_scan, gpu_scan_gated, gpu_step, normwise,
+                        oracle_outputs)
 from paper_2406_12580_gb300 import inputs as I
 
 torch = pytest.importorskip("torch")
@@ -261,3 +262,43 @@ def test_binding_rejects_host_tensors():
     x = torch.zeros(1, 4, 8)
     with pytest.raises(ValueError):
         blr_scan_fwd(Desc(1, 4, 8), x, x, x, None, x, None, x)
+
+
+# The gated layer's merge y = h SiLU(z) (Alg. 1): fused into the serial kernels
+# (many chains) and composed with the tiled kernels (few chains), both dtypes.
+GATED = [
+    dict(B=1, L=1, D=8),
+    dict(B=3, L=65, D=72, random_h0=True, random_dh_last=True),
+    dict(B=2, L=300, D=16, c=2.0, decay=(0.05, 0.95)),
+    dict(B=300, L=203, D=24, random_h0=True, random_dh_last=True),
+    dict(B=700, L=37, D=40, decay=(0.05, 0.95), c=0.5),
+    dict(B=260, L=1100, D=8, decay=(0.99, 0.9999), random_h0=True),
+]
+
+
+@pytest.mark.parametrize("io", [I.F32, I.BF16])
+@pytest.mark.parametrize("case", range(len(GATED)))
+def test_gated_small_shapes(io, case):
+    inp = I.make_scan_inputs(_cfg(io, 300 + case, gated=True, **GATED[case]))
+    buf = gpu_scan_gated(inp)
+    compare(inp, gpu_outputs(buf), oracle_outputs(inp))
+
+
+@pytest.mark.parametrize("k", [1, 2])
+def test_gated_config_full_oracle(k):
+    """The headline and train-shaped workloads gated, at full size."""
+    inp = I.make_scan_inputs(I.scaled(I.CONFIGS[k], gated=True))
+    buf = gpu_scan_gated(inp)
+    errs = compare(inp, gpu_outputs(buf), oracle_outputs(inp, threads=0))
+    print(f"gated config {k}: {errs}")
+
+
+def test_gated_long_sequence_sampled():
+    """The long-sequence workload gated (tiled kernels and the merge kernels),
+    on sampled channels."""
+    cfg = I.scaled(I.CONFIGS[4], gated=True)
+    inp = I.make_scan_inputs(cfg)
+    buf = gpu_scan_gated(inp)
+    dsel = _sampled_channels(cfg.D)
+    errs = compare(inp, gpu_outputs(buf, dsel), oracle_outputs(inp, dsel, threads=0))
+    print(f"gated config 4: {errs}")
