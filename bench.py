@@ -527,7 +527,73 @@ def other_workloads(flush, peak, dev, headline):
                              "frac": gbs / peak}
         del sbuf
     out["step_f32_graph"] = step_graph(flush, peak, dev)
+    for k in (1, 2):
+        out[f"gated_config{k}"] = gated_workload(k, flush, peak, dev)
     return out
+
+
+def gated_workload(k, flush, peak, dev, reps=20):
+    """Workload k with the gated layer's merge y = h SiLU(z) (Alg. 1): the fused
+    entry points against the plain scan followed by the merge as separate torch
+    elementwise operations (what a caller without the fused call would run)."""
+    import torch
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = I.scaled(I.CONFIGS[k], gated=True)
+    buf = ScanBuffers.from_inputs(I.make_scan_inputs(cfg), device=dev)
+    z, dy = buf.z, buf.dh
+    dh = torch.empty_like(dy)
+
+    def fused():
+        buf.fwd_gated()
+        e = torch.cuda.Event(enable_timing=True)
+        e.record()
+        buf.bwd_gated()
+        return e
+
+    def unfused():
+        buf.fwd()
+        y = buf.h * torch.nn.functional.silu(z)
+        e = torch.cuda.Event(enable_timing=True)
+        e.record()
+        sg = torch.sigmoid(z)
+        torch.mul(dy, z * sg, out=dh)
+        dz = dy * buf.h * (sg * (1 + z * (1 - sg)))
+        blr_scan_bwd_buf(buf, dh)
+        return e, y, dz
+
+    def blr_scan_bwd_buf(b, dh_):
+        from paper_2406_12580_gb300 import blr_scan_bwd
+        blr_scan_bwd(b.desc, dh_, b.dh_last, b.x, b.gl, b.lam, b.h0, b.dx, b.dgl, b.dlam, b.dh0,
+                     b.ws)
+
+    res = {}
+    for name, fn in (("fused", fused), ("unfused", unfused)):
+        for _ in range(3):
+            fn()
+        ev = []
+        for _ in range(reps):
+            flush()
+            e0, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            r = fn()
+            e2.record()
+            ev.append((e0, r[0] if isinstance(r, tuple) else r, e2))
+        torch.cuda.synchronize()
+        f = statistics.median(a.elapsed_time(b) for a, b, c in ev)
+        b = statistics.median(b.elapsed_time(c) for a, b, c in ev)
+        res[name] = {"fwd_ms": f, "bwd_ms": b}
+    n, ib = cfg.elements, io_bytes(cfg.io)
+    fu = res["fused"]
+    # compulsory bytes of the fused calls: fwd x, rho, iota, z in, y out (5 values);
+    # bwd dy, x, rho, iota, z in, dx, drho, diota, dz out (9 values)
+    gbs = n * 14 * ib / ((fu["fwd_ms"] + fu["bwd_ms"]) * 1e-3) / 1e9
+    return {"workload": cfg.name + ", gated (y = h SiLU(z))", "fused": res["fused"],
+            "unfused_scan_then_torch_merge": res["unfused"],
+            "fused_elements_per_s": n / ((fu["fwd_ms"] + fu["bwd_ms"]) * 1e-3),
+            "fused_speedup": (res["unfused"]["fwd_ms"] + res["unfused"]["bwd_ms"]) /
+                             (fu["fwd_ms"] + fu["bwd_ms"]),
+            "fused_gbs": gbs, "fused_frac": gbs / peak}
 
 
 def step_graph(flush, peak, dev, n_tok=8, reps=20):
