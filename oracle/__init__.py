@@ -13,6 +13,7 @@ Functions and the passages they follow:
   fwd(x, gl, lam, h0, c)            -> h, h_last             Sec. 3.2, Eq. linrnn
   bwd(dh, x, gl, lam, h0, dh_last)  -> dx, dgl, dlam, dh0    chain rule of Sec. 3.2 (not printed in the paper)
   step(h_prev, x, gl, lam, c)       -> h_t                   Sec. 1 / Sec. 4.3 (recurrent inference)
+  steps(h_prev, x, gl, lam, c)      -> h_seq, h_out         K recurrent steps per row (step, repeated)
   fwd_gated(x, gl, lam, z, h0, c)   -> y = h SiLU(z), h_last  Alg. 1 (the scan, then the merge H_y (x) SiLU(H_z))
   bwd_gated(dy, x, gl, lam, z, ...) -> dx, dgl, dlam, dh0, dz  chain rule through the merge, then bwd
 
@@ -154,6 +155,18 @@ class Oracle:
         h_t = np.empty((B, D))
         self._lib.blr_oracle_step(B, D, c, _ptr(h_prev), _ptr(x), _ptr(gl), _ptr(lam), _ptr(h_t))
         return h_t
+
+    def steps(self, h_prev, x, gl, lam, c: float = 1.0):
+        """K consecutive recurrent steps of every row: x (B, K, D), gl (B, K, 2D).
+        Returns (h_seq (B, K, D), h_out (B, D)); one call of step per step."""
+        x, gl = _f64(x), _f64(gl)
+        B, K, D = x.shape
+        h = _f64(h_prev, (B, D))
+        h_seq = np.empty((B, K, D))
+        for j in range(K):
+            h = self.step(h, x[:, j], gl[:, j], lam, c=c)
+            h_seq[:, j] = h
+        return h_seq, h
 
     def merge(self, h, z):
         """y = h SiLU(z), elementwise (Alg. 1, the merge of the two branches)."""

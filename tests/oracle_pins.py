@@ -14,7 +14,8 @@ the oracle disagrees with something the paper or mathematics fixes:
   * split / resume of the state;
   * the stability bound implied by alpha, beta in [0, 1] (Sec. 3.2);
   * central finite differences of every gradient, linearity of the gradient in
-    dh, and consistency of the single step with a length-1 scan;
+    dh, and consistency of the single step with a length-1 scan, of K steps
+    with a length-K scan and with the closed form of constant gates;
   * for the merge of the gated layer (Alg. 1, y = h SiLU(z)): SiLU's values and
     slope at 0 and its limits z -> +-inf, the reduction to the plain scan at
     the z where SiLU(z) = 1 (found by root finding on scipy's expit), and
@@ -338,6 +339,20 @@ def pin_step(orc):
     assert _rel(ht, 0.5 * h_prev + math.sqrt(3) / 4 * x[:, 0]) < 1e-15
 
 
+def pin_steps(orc):
+    rng = np.random.default_rng(26)
+    B, K, D = 4, 7, 5
+    x, gl, lam = _rand_problem(rng, B, K, D)
+    h_prev = rng.standard_normal((B, D))
+    h_seq, h_out = orc.steps(h_prev, x, gl, lam, c=1.3)
+    h, hl = orc.fwd(x, gl, lam, h_prev, c=1.3)  # K steps are a length-K scan from h_prev
+    assert np.array_equal(h_seq, h) and np.array_equal(h_out, hl)
+    # closed form: c = 2, Lambda = rho = iota = 0 -> alpha = 1/2, beta = sqrt(3)/4 every step
+    _, h_out = orc.steps(h_prev, x, np.zeros((B, K, 2 * D)), np.zeros(D), c=2.0)
+    want = 0.5 ** K * h_prev + sum(0.5 ** (K - 1 - j) * math.sqrt(3) / 4 * x[:, j] for j in range(K))
+    assert _rel(h_out, want) < 1e-14
+
+
 # ----------------------------------------------------- the gated layer's merge
 
 
@@ -427,6 +442,7 @@ ALL_PINS = [
     pin_finite_differences,
     pin_gradient_linearity,
     pin_step,
+    pin_steps,
     pin_merge_limits,
     pin_merge_unit_gate,
     pin_gated_finite_differences,
