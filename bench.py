@@ -527,9 +527,43 @@ def other_workloads(flush, peak, dev, headline):
                              "frac": gbs / peak}
         del sbuf
     out["step_f32_graph"] = step_graph(flush, peak, dev)
+    for io in ("f32", "bf16"):
+        out[f"steps_k8_{io}"] = steps_workload(io, flush, peak, dev)
     for k in (1, 2):
         out[f"gated_config{k}"] = gated_workload(k, flush, peak, dev)
     return out
+
+
+def steps_workload(io, flush, peak, dev, B=65536, K=8, D=64, reps=20):
+    """K = 8 recurrent steps per row in one call (blr_steps), state and I/O in
+    the same dtype, per-step states not written: compulsory bytes per (row,
+    channel) are the state in and out plus K x (x, rho, iota)."""
+    import torch
+    from paper_2406_12580_gb300 import blr_steps
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import io_code, to_device, torch_io_dtype
+    cfg = I.ScanConfig(f"{K} recurrent steps B={B} D={D} {io}", B, K, D, io, seed=6,
+                       fwd_only=True, random_h0=True)
+    inp = I.make_scan_inputs(cfg)
+    x, gl = to_device(inp.io_array("x"), io, dev), to_device(inp.io_array("gl"), io, dev)
+    lam = to_device(inp.lam, "f32", dev)
+    h = torch.from_numpy(inp.h0).to(dev).to(torch_io_dtype(io))
+    code = io_code(io)
+    for _ in range(3):
+        blr_steps(B, K, D, code, code, 1.0, h, x, gl, lam, h)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(reps)]
+    for e0, e1 in ev:
+        flush()
+        e0.record()
+        blr_steps(B, K, D, code, code, 1.0, h, x, gl, lam, h)
+        e1.record()
+    torch.cuda.synchronize()
+    ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+    ib = io_bytes(io)
+    gbs = B * D * (2 + 3 * K) * ib / (ms * 1e-3) / 1e9
+    return {"workload": cfg.name + " in one call", "ms": ms,
+            "steps_per_s": B * D * K / (ms * 1e-3), "gbs": gbs, "frac": gbs / peak}
 
 
 def gated_workload(k, flush, peak, dev, reps=20):

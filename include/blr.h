@@ -197,6 +197,28 @@ BLR_API blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const f
                     blr_stream_t stream);
 
 /*
+ * K consecutive recurrent-inference steps for a batch of states: serving K new
+ * behaviors per user in one call (the low-cost recurrent inference of Sec. 1
+ * and Sec. 4.3, K times):
+ *   h_j = alpha_j * h_{j-1} + beta_j * x_j,  j = 1..K,  h_0 = h_prev.
+ * io          dtype of x, gate_logits and h_seq
+ * state       dtype of h_prev and h_out: BLR_F32, or BLR_BF16 to halve the state's
+ *             memory (the K steps run in float32; h_out is rounded to
+ *             nearest-even once)
+ * h_prev      (B, D) state dtype
+ * x           (B, K, D) io dtype, the K new inputs of every row, oldest first
+ * gate_logits (B, K, 2D) io dtype, [rho | iota] of every step
+ * lambda      (D) float32
+ * h_out       (B, D) state dtype, the state after step K; may alias h_prev exactly
+ * h_seq       (B, K, D) io dtype or NULL: the state after every step
+ * K == 0 copies h_prev to h_out. Needs no workspace. Pointers 16-byte aligned;
+ * no output may overlap an input except h_out == h_prev.
+ */
+BLR_API blr_status blr_steps(int64_t B, int64_t K, int64_t D, blr_dtype io, blr_dtype state, float c,
+                             const void* h_prev, const void* x, const void* gate_logits,
+                             const float* lambda, void* h_out, void* h_seq, blr_stream_t stream);
+
+/*
  * Synchronises `stream`, then reads the error word that the kernels of
  * earlier calls on this workspace recorded: BLR_OK, BLR_ERR_TIMEOUT or
  * BLR_ERR_WORKSPACE (BLR_ERR_CUDA if the read itself fails). The word is

@@ -12,6 +12,7 @@ there is no CPU path.
     blr_scan_fwd(desc, x, gate_logits, lam, h0, h, h_last, ws)
     blr_scan_bwd(desc, dh, dh_last, x, gate_logits, lam, h0, dx, dgate_logits, dlam, dh0, ws)
     blr_step(B, D, BLR_F32, 1.0, h_prev, x_t, gate_logits_t, lam, h_t)
+    blr_steps(B, K, D, BLR_BF16, BLR_BF16, 1.0, h_prev, x, gate_logits, lam, h_out, h_seq)
 
 The gated recurrent layer's merge y = h SiLU(z) (Alg. 1) fused into the scan:
 
@@ -32,6 +33,7 @@ __all__ = [
     "BLR_F32", "BLR_BF16", "Desc", "BLRError", "blr_workspace_bytes", "blr_scan_fwd",
     "blr_scan_bwd", "blr_step", "blr_workspace_status", "blr_status_string",
     "blr_selftest_wait_timeout", "blr_scan_fwd_noalloc", "blr_scan_fwd_gated", "blr_scan_bwd_gated",
+    "blr_steps",
     "BDLRUScan", "library_loaded",
 ]
 
@@ -146,6 +148,14 @@ def blr_step(B, D, io, c, h_prev, x_t, gate_logits_t, lam, h_t, stream=None):
                            _ptr(gate_logits_t, "gate_logits_t"), _ptr(lam, "lambda"),
                            _ptr(h_t, "h_t"), _stream(stream)),
            "blr_step")
+
+
+def blr_steps(B, K, D, io, state, c, h_prev, x, gate_logits, lam, h_out, h_seq=None, stream=None):
+    """K recurrent steps per row (state dtype `state`, BLR_F32 or BLR_BF16)."""
+    _check(load().blr_steps(B, K, D, io, state, c, _ptr(h_prev, "h_prev"), _ptr(x, "x"),
+                            _ptr(gate_logits, "gate_logits"), _ptr(lam, "lambda"),
+                            _ptr(h_out, "h_out"), _ptr(h_seq, "h_seq"), _stream(stream)),
+           "blr_steps")
 
 
 def blr_workspace_status(desc, ws, stream=None) -> int:

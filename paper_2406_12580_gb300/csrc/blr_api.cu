@@ -621,6 +621,54 @@ blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_
   return cuda_check(cudaGetLastError(), "launch step_kernel");
 }
 
+blr_status blr_steps(int64_t B, int64_t K, int64_t D, blr_dtype io, blr_dtype state, float c,
+                     const void* h_prev, const void* x, const void* gate_logits,
+                     const float* lambda, void* h_out, void* h_seq, blr_stream_t stream) {
+  if (B < 0 || K < 0 || D < 0)
+    return fail(BLR_ERR_INVALID_ARG, "negative size B=%lld K=%lld D=%lld", (long long)B, (long long)K,
+                (long long)D);
+  if (io != BLR_F32 && io != BLR_BF16) return fail(BLR_ERR_INVALID_ARG, "unknown io dtype %d", (int)io);
+  if (state != BLR_F32 && state != BLR_BF16)
+    return fail(BLR_ERR_INVALID_ARG, "unknown state dtype %d", (int)state);
+  if (!(c > 0.0f) || !isfinite(c)) return fail(BLR_ERR_INVALID_ARG, "c must be finite and > 0");
+  if (D % 8 != 0) return fail(BLR_ERR_UNSUPPORTED, "D=%lld is not a multiple of 8", (long long)D);
+  if (B == 0 || D == 0) return BLR_OK;
+  if (D > (int64_t)1 << 24 || B > (int64_t)1 << 40 || K > (int64_t)1 << 40 ||
+      (double)B * (double)K * (double)D > 1e18)
+    return fail(BLR_ERR_UNSUPPORTED, "problem too large");
+  BLR_TRY(need(h_prev, "h_prev", 16));
+  BLR_TRY(need(h_out, "h_out", 16));
+  BLR_TRY(need(lambda, "lambda", 16));
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (K == 0) {  // no step: the state is unchanged
+    if (h_out == h_prev) return BLR_OK;
+    const size_t bytes = (size_t)B * (size_t)D * (state == BLR_F32 ? 4 : 2);
+    return cuda_check(cudaMemcpyAsync(h_out, h_prev, bytes, cudaMemcpyDeviceToDevice, st),
+                      "copy h_prev to h_out");
+  }
+  BLR_TRY(need(x, "x", 16));
+  BLR_TRY(need(gate_logits, "gate_logits", 16));
+  BLR_TRY(optional(h_seq, "h_seq", 16));
+  const int vec = io == BLR_F32 ? 4 : 8;
+  const int64_t threads = B * (D / vec);
+  const int64_t blocks = (threads + 255) / 256;
+  if (blocks >= ((int64_t)1 << 31)) return fail(BLR_ERR_UNSUPPORTED, "grid too large");
+  blr::StepsArgs a{B, K, D, c, h_prev, x, gate_logits, lambda, h_out, h_seq};
+  using bf = __nv_bfloat16;
+  if (io == BLR_F32) {
+    if (state == BLR_F32)
+      blr::steps_kernel<float, float, 4, blr::MathPrecise><<<(unsigned)blocks, 256, 0, st>>>(a);
+    else
+      blr::steps_kernel<float, bf, 4, blr::MathPrecise><<<(unsigned)blocks, 256, 0, st>>>(a);
+  } else {
+    if (state == BLR_F32)
+      blr::steps_kernel<bf, float, 8, blr::MathFast><<<(unsigned)blocks, 256, 0, st>>>(a);
+    else
+      blr::steps_kernel<bf, bf, 8, blr::MathFast><<<(unsigned)blocks, 256, 0, st>>>(a);
+  }
+  return cuda_check(cudaGetLastError(), "launch steps_kernel");
+}
+
 blr_status blr_workspace_status(const blr_desc* desc, const void* ws, size_t ws_bytes,
                                 blr_stream_t stream) {
   Plan plan;

@@ -995,6 +995,95 @@ __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
   }
 }
 
+// ------------------------------------------------------- K recurrent steps
+//
+// h_j = alpha_j h_{j-1} + beta_j x_j for j = 1..K and every (row, channel), from
+// h_0 = h_prev: a thread owns VEC channels of one row and walks its K steps
+// serially with the state in float32 registers, whatever the state dtype in
+// memory (a bfloat16 state is rounded once, when it is stored). The loads of
+// kStepsAhead steps are issued before the first of them is used.
+
+struct StepsArgs {
+  int64_t B, K, D;
+  float c;
+  const void* h_prev;  // (B, D), state dtype
+  const void* x;       // (B, K, D), io dtype
+  const void* gl;      // (B, K, 2D), io dtype
+  const float* lambda;
+  void* h_out;         // (B, D), state dtype
+  void* h_seq;         // (B, K, D), io dtype, or NULL
+};
+
+constexpr int kStepsAhead = 4;
+
+template <typename S, int VEC>
+__device__ __forceinline__ void load_state(const S* p, float (&h)[VEC]) {
+  if constexpr (sizeof(S) == 4)
+    load_f32<VEC>(reinterpret_cast<const float*>(p), h);
+  else
+    Io<__nv_bfloat16, VEC>::unpack(Io<__nv_bfloat16, VEC>::load_raw(p), h);
+}
+template <typename S, int VEC>
+__device__ __forceinline__ void store_state(S* p, const float (&h)[VEC]) {
+  if constexpr (sizeof(S) == 4) {
+#pragma unroll
+    for (int j = 0; j < VEC; j += 4)
+      *reinterpret_cast<float4*>(reinterpret_cast<float*>(p) + j) =
+          make_float4(h[j], h[j + 1], h[j + 2], h[j + 3]);
+  } else {
+    Io<__nv_bfloat16, VEC>::store(p, h);
+  }
+}
+
+template <typename T, typename S, int VEC, class M>
+__global__ void __launch_bounds__(256) steps_kernel(const StepsArgs a) {
+  using IO = Io<T, VEC>;
+  using Raw = typename IO::Raw;
+  const int64_t nv = a.D / VEC;
+  const int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (idx >= a.B * nv) return;
+  const int64_t b = idx / nv;
+  const int64_t d0 = (idx - b * nv) * VEC;
+  float k[VEC], h[VEC];
+#pragma unroll
+  for (int v = 0; v < VEC; ++v) k[v] = decay_rate(a.c, a.lambda[d0 + v]);
+  load_state<S, VEC>(static_cast<const S*>(a.h_prev) + b * a.D + d0, h);
+  const T* x = static_cast<const T*>(a.x) + b * a.K * a.D + d0;
+  const T* gl = static_cast<const T*>(a.gl) + b * a.K * 2 * a.D + d0;
+  T* hs = a.h_seq != nullptr ? static_cast<T*>(a.h_seq) + b * a.K * a.D + d0 : nullptr;
+  for (int64_t j0 = 0; j0 < a.K; j0 += kStepsAhead) {
+    Raw rx[kStepsAhead], rr[kStepsAhead], ri[kStepsAhead];
+#pragma unroll
+    for (int u = 0; u < kStepsAhead; ++u) {
+      const int64_t j = j0 + u;
+      if (j < a.K) {
+        rx[u] = IO::load_raw(x + j * a.D);
+        rr[u] = IO::load_raw(gl + j * 2 * a.D);
+        ri[u] = IO::load_raw(gl + j * 2 * a.D + a.D);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kStepsAhead; ++u) {
+      const int64_t j = j0 + u;
+      if (j < a.K) {
+        float xv[VEC], rv[VEC], iv[VEC];
+        IO::unpack(rx[u], xv);
+        IO::unpack(rr[u], rv);
+        IO::unpack(ri[u], iv);
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) {
+          const float r = M::sigmoid(rv[v]);
+          const float i = M::sigmoid(iv[v]);
+          const float e = M::expm1_any(k[v] * r);
+          h[v] = fmaf(1.0f + e, h[v], M::sqrt(-e * (2.0f + e)) * i * xv[v]);
+        }
+        if (hs != nullptr) IO::store(hs + j * a.D, h);
+      }
+    }
+  }
+  store_state<S, VEC>(static_cast<S*>(a.h_out) + b * a.D + d0, h);
+}
+
 // ------------------------------------------------------------ bounded-wait test
 
 __global__ void selftest_wait_kernel(const uint32_t* flag, uint32_t* err, uint64_t timeout_ns) {

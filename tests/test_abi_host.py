@@ -143,6 +143,23 @@ def test_gated_validation(lib):
     assert b"dy is NULL" in lib.blr_last_error_string()
 
 
+def test_steps_validation(lib):
+    f = lambda B, K, Dd, io=0, st=0, c=1.0, hp=FAKE, x=FAKE, gl=FAKE, lam=FAKE, ho=FAKE, hs=None: \
+        lib.blr_steps(B, K, Dd, io, st, c, hp, x, gl, lam, ho, hs, None)  # noqa: E731
+    assert f(-1, 2, 8) == _lib.BLR_ERR_INVALID_ARG
+    assert f(4, -2, 8) == _lib.BLR_ERR_INVALID_ARG
+    assert f(4, 2, 8, io=2) == _lib.BLR_ERR_INVALID_ARG
+    assert f(4, 2, 8, st=5) == _lib.BLR_ERR_INVALID_ARG
+    assert f(4, 2, 8, c=0.0) == _lib.BLR_ERR_INVALID_ARG
+    assert f(4, 2, 12) == _lib.BLR_ERR_UNSUPPORTED
+    for name in ("hp", "x", "gl", "lam", "ho"):
+        assert f(4, 2, 8, **{name: None}) == _lib.BLR_ERR_INVALID_ARG, name
+        assert f(4, 2, 8, **{name: FAKE + 8}) == _lib.BLR_ERR_INVALID_ARG, name
+    assert f(4, 2, 8, hs=FAKE + 4) == _lib.BLR_ERR_INVALID_ARG
+    assert f(0, 2, 8, hp=None, x=None, gl=None, lam=None, ho=None) == _lib.BLR_OK
+    assert f(4, 0, 8, hp=FAKE, x=None, gl=None, ho=FAKE) == _lib.BLR_OK  # K = 0, in place: nothing to do
+
+
 def test_step_validation(lib):
     f = lib.blr_step
     assert f(-1, 8, 0, 1.0, FAKE, FAKE, FAKE, FAKE, FAKE, None) == _lib.BLR_ERR_INVALID_ARG

@@ -302,3 +302,44 @@ def test_gated_long_sequence_sampled():
     dsel = _sampled_channels(cfg.D)
     errs = compare(inp, gpu_outputs(buf, dsel), oracle_outputs(inp, dsel, threads=0))
     print(f"gated config 4: {errs}")
+
+
+# K recurrent steps per row (blr_steps): io and state dtypes crossed, with and
+# without the per-step states, the last state written over the first.
+STEPS = [dict(B=1, L=1, D=8), dict(B=3, L=5, D=72), dict(B=1000, L=16, D=64, c=2.0),
+         dict(B=65536, L=8, D=64, decay=(0.99, 0.9999))]
+
+
+def _bf16_round(a):
+    return I.bf16_bits_to_f32(I.round_to_bf16(a)).reshape(a.shape)
+
+
+@pytest.mark.parametrize("state", [I.F32, I.BF16])
+@pytest.mark.parametrize("io", [I.F32, I.BF16])
+@pytest.mark.parametrize("case", range(len(STEPS)))
+def test_steps(case, io, state):
+    import oracle
+    from paper_2406_12580_gb300 import blr_steps
+    from paper_2406_12580_gb300.device import io_code, to_device, torch_io_dtype
+    cfg = _cfg(io, 500 + case, random_h0=True, fwd_only=True, **STEPS[case])
+    inp = I.make_scan_inputs(cfg)
+    B, K, D = cfg.B, cfg.L, cfg.D
+    h_prev = inp.h0 if state == I.F32 else _bf16_round(inp.h0)
+    x, gl = to_device(inp.io_array("x"), io, "cuda"), to_device(inp.io_array("gl"), io, "cuda")
+    lam = to_device(inp.lam, I.F32, "cuda")
+    h = torch.from_numpy(h_prev.astype(np.float32)).cuda().to(torch_io_dtype(state))
+    h_seq = torch.empty(B, K, D, dtype=torch_io_dtype(io), device="cuda")
+    blr_steps(B, K, D, io_code(io), io_code(state), cfg.c, h, x, gl, lam, h, h_seq)  # in place
+    torch.cuda.synchronize()
+    want_seq, want_out = oracle.load().steps(h_prev, inp.x, inp.gl, inp.lam, c=cfg.c)
+    assert normwise(h_seq.float().cpu().numpy(), want_seq) <= TOL[io]
+    tol_out = TOL[I.F32] if (io == I.F32 and state == I.F32) else TOL[I.BF16]
+    assert normwise(h.float().cpu().numpy(), want_out) <= tol_out
+    # without the per-step states, into a separate output; K = 0 copies the state
+    h2 = torch.from_numpy(h_prev.astype(np.float32)).cuda().to(torch_io_dtype(state))
+    out = torch.empty_like(h2)
+    blr_steps(B, K, D, io_code(io), io_code(state), cfg.c, h2, x, gl, lam, out, None)
+    blr_steps(B, 0, D, io_code(io), io_code(state), cfg.c, out, None, None, lam, h2, None)
+    torch.cuda.synchronize()
+    assert torch.equal(out, h)
+    assert torch.equal(h2, out)
