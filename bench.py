@@ -531,6 +531,7 @@ def other_workloads(flush, peak, dev, headline):
         out[f"steps_k8_{io}"] = steps_workload(io, flush, peak, dev)
     for k in (1, 2):
         out[f"gated_config{k}"] = gated_workload(k, flush, peak, dev)
+    out["gated_layer_train_step"] = layer_workload(flush, dev)
     return out
 
 
@@ -564,6 +565,53 @@ def steps_workload(io, flush, peak, dev, B=65536, K=8, D=64, reps=20):
     gbs = B * D * (2 + 3 * K) * ib / (ms * 1e-3) / 1e9
     return {"workload": cfg.name + " in one call", "ms": ms,
             "steps_per_s": B * D * K / (ms * 1e-3), "gbs": gbs, "frac": gbs / peak}
+
+
+def layer_workload(flush, dev, B=256, L=200, D=64, E=2, reps=10):
+    """One training step (forward and backward) of the gated recurrent layer
+    of Alg. 1 (layer.GatedRecurrentLayer: torch GEMMs and convolution, the scan
+    and merge on the library's kernels) against the same layer with the scan as
+    a step-by-step torch loop on the GPU (a serial scan)."""
+    import torch
+    from paper_2406_12580_gb300.layer import GatedRecurrentLayer
+    torch.manual_seed(0)
+    layer = GatedRecurrentLayer(D, expand=E, device=dev)
+    h = torch.randn(B, L, D, device=dev, requires_grad=True)
+    g = torch.randn(B, L, D, device=dev)
+
+    def serial_forward(x_in):
+        hx, hz = layer.in_proj(x_in).split(layer.ed, dim=-1)
+        xc = layer.conv(hx.transpose(1, 2))[..., :L].transpose(1, 2)
+        x = torch.nn.functional.silu(xc)
+        rho, iota = layer.gate_proj(x).split(layer.ed, dim=-1)
+        alpha = torch.exp(-torch.nn.functional.softplus(layer.lam) * torch.sigmoid(rho))
+        beta = torch.sqrt(1.0 - alpha * alpha) * torch.sigmoid(iota)
+        state = torch.zeros(B, layer.ed, device=dev)
+        hs = []
+        for t in range(L):
+            state = alpha[:, t] * state + beta[:, t] * x[:, t]
+            hs.append(state)
+        return layer.out_proj(torch.stack(hs, dim=1) * torch.nn.functional.silu(hz))
+
+    res = {}
+    for name, fwd in (("fused_kernels", layer), ("serial_torch_scan", serial_forward)):
+        n = reps if name == "fused_kernels" else max(2, reps // 5)
+        for _ in range(2):
+            (fwd(h) * g).sum().backward()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(n)]
+        for e0, e1 in ev:
+            flush()
+            e0.record()
+            (fwd(h) * g).sum().backward()
+            e1.record()
+        torch.cuda.synchronize()
+        res[name] = statistics.median(a.elapsed_time(b) for a, b in ev)
+    return {"workload": f"gated recurrent layer (Alg. 1) d_model={D} E={E} B={B} L={L} f32, "
+                        "forward + backward", "ms_fused_kernels": res["fused_kernels"],
+            "ms_serial_torch_scan": res["serial_torch_scan"],
+            "tokens_per_s": B * L / (res["fused_kernels"] * 1e-3),
+            "serial_over_fused": res["serial_torch_scan"] / res["fused_kernels"]}
 
 
 def gated_workload(k, flush, peak, dev, reps=20):
