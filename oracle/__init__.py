@@ -14,6 +14,8 @@ Functions and the passages they follow:
   bwd(dh, x, gl, lam, h0, dh_last)  -> dx, dgl, dlam, dh0    chain rule of Sec. 3.2 (not printed in the paper)
   step(h_prev, x, gl, lam, c)       -> h_t                   Sec. 1 / Sec. 4.3 (recurrent inference)
   steps(h_prev, x, gl, lam, c)      -> h_seq, h_out         K recurrent steps per row (step, repeated)
+  fwd_varlen / bwd_varlen(lengths, ...)                     per-row lengths: row b is its last lengths[b]
+                                                            steps (Sec. 3.3's left padding, not read)
   fwd_gated(x, gl, lam, z, h0, c)   -> y = h SiLU(z), h_last  Alg. 1 (the scan, then the merge H_y (x) SiLU(H_z))
   bwd_gated(dy, x, gl, lam, z, ...) -> dx, dgl, dlam, dh0, dz  chain rule through the merge, then bwd
 
@@ -167,6 +169,50 @@ class Oracle:
             h = self.step(h, x[:, j], gl[:, j], lam, c=c)
             h_seq[:, j] = h
         return h_seq, h
+
+    def fwd_varlen(self, lengths, x, gl, lam, h0=None, c: float = 1.0, threads: int = 1):
+        """Row b is a sequence of its last lengths[b] steps (rows [L - len, L));
+        the rows before it are not part of it. Returns (h, h_last) with h NaN on
+        those rows (nothing is computed there)."""
+        x, gl, lam = _f64(x), _f64(gl), _f64(lam)
+        B, L, D = self._dims(x, gl, lam)
+        h = np.full((B, L, D), np.nan)
+        h_last = np.empty((B, D))
+        for b in range(B):
+            t0 = L - int(lengths[b])
+            hb0 = None if h0 is None else _f64(h0)[b:b + 1]
+            if t0 == L:
+                h_last[b] = 0.0 if hb0 is None else hb0[0]
+                continue
+            hb, hl = self.fwd(x[b:b + 1, t0:], gl[b:b + 1, t0:], lam, hb0, c=c, threads=threads)
+            h[b, t0:] = hb[0]
+            h_last[b] = hl[0]
+        return h, h_last
+
+    def bwd_varlen(self, lengths, dh, x, gl, lam, h0=None, dh_last=None, c: float = 1.0,
+                   threads: int = 1):
+        """Backward of fwd_varlen: (dx, dgl, dlam, dh0), dx and dgl NaN on the rows
+        before each sequence; dh there is not read."""
+        x, gl, lam = _f64(x), _f64(gl), _f64(lam)
+        B, L, D = self._dims(x, gl, lam)
+        dh = _f64(dh, (B, L, D))
+        dx = np.full((B, L, D), np.nan)
+        dgl = np.full((B, L, 2 * D), np.nan)
+        dlam = np.zeros(D)
+        dh0 = np.empty((B, D))
+        for b in range(B):
+            t0 = L - int(lengths[b])
+            dl = np.zeros(D) if dh_last is None else _f64(dh_last)[b]
+            if t0 == L:
+                dh0[b] = dl
+                continue
+            hb0 = None if h0 is None else _f64(h0)[b:b + 1]
+            g = self.bwd(dh[b:b + 1, t0:], x[b:b + 1, t0:], gl[b:b + 1, t0:], lam, hb0,
+                         dl[None], c=c, threads=threads)
+            dx[b, t0:], dgl[b, t0:] = g[0][0], g[1][0]
+            dlam += g[2]
+            dh0[b] = g[3][0]
+        return dx, dgl, dlam, dh0
 
     def merge(self, h, z):
         """y = h SiLU(z), elementwise (Alg. 1, the merge of the two branches)."""

@@ -10,7 +10,8 @@ the oracle disagrees with something the paper or mathematics fixes:
   * the O(L^2) unrolled sum, with gates from library primitives (scipy's expit,
     numpy's logaddexp), on tiny inputs;
   * the paper's two-tree parallel scan (Sec. 3.3, Fig. "scan") at T = 8;
-  * zero left-padding invariance (Sec. 3.3, embedding padding);
+  * zero left-padding invariance (Sec. 3.3, embedding padding), and per-row
+    lengths against the zero-padded scan;
   * split / resume of the state;
   * the stability bound implied by alpha, beta in [0, 1] (Sec. 3.2);
   * central finite differences of every gradient, linearity of the gradient in
@@ -353,6 +354,60 @@ def pin_steps(orc):
     assert _rel(h_out, want) < 1e-14
 
 
+def pin_varlen_is_zero_left_padding(orc):
+    # Sec. 3.3: sequences left-padded with zero rows scan to the same states (h0
+    # = 0); so a per-row length that skips the padding must give the padded
+    # scan's values on the real rows, and the same gate and Lambda gradients
+    # when dh is zero on the padding. dh0 differs by the padding's decay.
+    rng = np.random.default_rng(27)
+    B, L, D, c = 4, 12, 3, 1.2
+    x, gl, lam = _rand_problem(rng, B, L, D)
+    lengths = np.array([12, 7, 1, 0])
+    dh = rng.standard_normal((B, L, D))
+    dh_last = rng.standard_normal((B, D))
+    for b, n in enumerate(lengths):
+        x[b, :L - n] = 0.0
+        gl[b, :L - n] = 0.0
+        dh[b, :L - n] = 0.0
+    h, hl = orc.fwd(x, gl, lam, None, c=c)
+    hv, hlv = orc.fwd_varlen(lengths, x, gl, lam, None, c=c)
+    real = ~np.isnan(hv)
+    assert np.array_equal(real, np.broadcast_to((np.arange(L)[None, :, None] >= (L - lengths)[:, None, None]), real.shape))
+    assert _rel(hv[real], h[real]) < 1e-14 and _rel(hlv, hl) < 1e-14
+    dx, dgl, dlam, dh0 = orc.bwd(dh, x, gl, lam, None, dh_last, c=c)
+    dxv, dglv, dlamv, dh0v = orc.bwd_varlen(lengths, dh, x, gl, lam, None, dh_last, c=c)
+    assert _rel(dxv[real], dx[real]) < 1e-13
+    real2 = np.concatenate([real, real], axis=2)
+    assert _rel(dglv[real2], dgl[real2]) < 1e-13
+    assert _rel(dlamv, dlam) < 1e-13
+    # padding rows have x = rho = iota = 0: alpha = exp(c * k / 2) each, k = -softplus
+    apad = np.exp(-c * np.logaddexp(0.0, lam) * 0.5)
+    for b, n in enumerate(lengths):
+        assert _rel(dh0[b], dh0v[b] * apad ** (L - n)) < 1e-13
+
+
+def pin_varlen_full_and_empty(orc):
+    rng = np.random.default_rng(28)
+    B, L, D = 3, 9, 4
+    x, gl, lam = _rand_problem(rng, B, L, D)
+    h0 = rng.standard_normal((B, D))
+    dh = rng.standard_normal((B, L, D))
+    full = np.full(B, L)
+    h, hl = orc.fwd(x, gl, lam, h0)
+    hv, hlv = orc.fwd_varlen(full, x, gl, lam, h0)
+    assert np.array_equal(h, hv) and np.array_equal(hl, hlv)
+    g = orc.bwd(dh, x, gl, lam, h0, None)
+    gv = orc.bwd_varlen(full, dh, x, gl, lam, h0, None)
+    for a_, b_ in zip(g, gv):
+        assert _rel(b_, a_) < 1e-14
+    # empty sequences: the state is h0, its gradient dh_last, nothing else moves
+    dh_last = rng.standard_normal((B, D))
+    _, hl0 = orc.fwd_varlen(np.zeros(B, dtype=int), x, gl, lam, h0)
+    assert np.array_equal(hl0, h0)
+    _, _, dlam0, dh00 = orc.bwd_varlen(np.zeros(B, dtype=int), dh, x, gl, lam, h0, dh_last)
+    assert np.array_equal(dh00, dh_last) and np.array_equal(dlam0, np.zeros(D))
+
+
 # ----------------------------------------------------- the gated layer's merge
 
 
@@ -443,6 +498,8 @@ ALL_PINS = [
     pin_gradient_linearity,
     pin_step,
     pin_steps,
+    pin_varlen_is_zero_left_padding,
+    pin_varlen_full_and_empty,
     pin_merge_limits,
     pin_merge_unit_gate,
     pin_gated_finite_differences,
