@@ -147,6 +147,33 @@ BLR_API blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const floa
                         blr_stream_t stream);
 
 /*
+ * Forward and backward scans of a batch whose rows carry their own lengths:
+ * row b's sequence is its last lengths[b] steps, rows [L - lengths[b], L) (the
+ * left-padded layout of Sec. 3.3's embedding padding). The rows before it are
+ * padding: x, gate_logits and dh there are never read, and h, dx and
+ * dgate_logits there are never written. The state before the sequence's
+ * first step is h0[b] (0 when h0 is NULL); h_last[b] is the state after step
+ * L - 1 (h0[b] for an empty row); dh0[b] is the gradient of the state before
+ * the first step; dlambda sums over the sequences' steps only.
+ * lengths     (B) int32 device array, 4-byte aligned; values outside [0, L]
+ *             are clamped
+ * Other arguments, the workspace (sized by blr_workspace_bytes for L) and the
+ * errors as blr_scan_fwd / blr_scan_bwd; the backward's ws must come from a
+ * blr_scan_fwd_varlen with the same lengths. Work and traffic scale with the
+ * rows' lengths on problems served by the serial kernels (at least 256
+ * chains); the tiled kernels still stream the padding and mask it.
+ */
+BLR_API blr_status blr_scan_fwd_varlen(const blr_desc* desc, const int32_t* lengths, const void* x,
+                                       const void* gate_logits, const float* lambda, const float* h0,
+                                       void* h, float* h_last, void* ws, size_t ws_bytes,
+                                       blr_stream_t stream);
+BLR_API blr_status blr_scan_bwd_varlen(const blr_desc* desc, const int32_t* lengths, const void* dh,
+                                       const float* dh_last, const void* x, const void* gate_logits,
+                                       const float* lambda, const float* h0, void* dx,
+                                       void* dgate_logits, float* dlambda, float* dh0, void* ws,
+                                       size_t ws_bytes, blr_stream_t stream);
+
+/*
  * Forward scan fused with the merge of the gated recurrent layer (Alg. 1,
  * H'_y = H_y (x) SiLU(H_z), the line after the BD-LRU):
  *   y[b,t,d] = h[b,t,d] * SiLU(z[b,t,d]),   SiLU(z) = z * sigmoid(z),

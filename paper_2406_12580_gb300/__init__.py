@@ -33,7 +33,7 @@ __all__ = [
     "BLR_F32", "BLR_BF16", "Desc", "BLRError", "blr_workspace_bytes", "blr_scan_fwd",
     "blr_scan_bwd", "blr_step", "blr_workspace_status", "blr_status_string",
     "blr_selftest_wait_timeout", "blr_scan_fwd_noalloc", "blr_scan_fwd_gated", "blr_scan_bwd_gated",
-    "blr_steps",
+    "blr_steps", "blr_scan_fwd_varlen", "blr_scan_bwd_varlen",
     "BDLRUScan", "library_loaded",
 ]
 
@@ -119,6 +119,28 @@ def blr_scan_bwd(desc, dh, dh_last, x, gate_logits, lam, h0, dx, dgate_logits, d
                                _ptr(dlam, "dlambda"), _ptr(dh0, "dh0"), _ptr(ws, "ws"), ws_bytes,
                                _stream(stream)),
            "blr_scan_bwd")
+
+
+def blr_scan_fwd_varlen(desc, lengths, x, gate_logits, lam, h0, h, h_last, ws, stream=None):
+    """blr_scan_fwd for rows of their own lengths (int32, on the device)."""
+    ws_bytes = ws.numel() if ws is not None and not isinstance(ws, int) else blr_workspace_bytes(desc)
+    _check(load().blr_scan_fwd_varlen(ctypes.byref(desc), _ptr(lengths, "lengths"), _ptr(x, "x"),
+                                      _ptr(gate_logits, "gate_logits"), _ptr(lam, "lambda"),
+                                      _ptr(h0, "h0"), _ptr(h, "h"), _ptr(h_last, "h_last"),
+                                      _ptr(ws, "ws"), ws_bytes, _stream(stream)),
+           "blr_scan_fwd_varlen")
+
+
+def blr_scan_bwd_varlen(desc, lengths, dh, dh_last, x, gate_logits, lam, h0, dx, dgate_logits,
+                        dlam, dh0, ws, stream=None):
+    ws_bytes = ws.numel() if ws is not None and not isinstance(ws, int) else blr_workspace_bytes(desc)
+    _check(load().blr_scan_bwd_varlen(ctypes.byref(desc), _ptr(lengths, "lengths"), _ptr(dh, "dh"),
+                                      _ptr(dh_last, "dh_last"), _ptr(x, "x"),
+                                      _ptr(gate_logits, "gate_logits"), _ptr(lam, "lambda"),
+                                      _ptr(h0, "h0"), _ptr(dx, "dx"),
+                                      _ptr(dgate_logits, "dgate_logits"), _ptr(dlam, "dlambda"),
+                                      _ptr(dh0, "dh0"), _ptr(ws, "ws"), ws_bytes, _stream(stream)),
+           "blr_scan_bwd_varlen")
 
 
 def blr_scan_fwd_gated(desc, x, gate_logits, lam, h0, z, y, h_last, ws, stream=None):

@@ -44,6 +44,9 @@ SIGNATURES = {
     "blr_last_error_string": (ctypes.c_char_p, []),
     "blr_selftest_wait_timeout": (_ST, [_DESC_P, _VP, _SZ, ctypes.c_uint64, _VP]),
     "blr_scan_fwd_noalloc": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
+    "blr_scan_fwd_varlen": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]),
+    "blr_scan_bwd_varlen": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
+                                  _VP, _SZ, _VP]),
     "blr_steps": (_ST, [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
                         ctypes.c_float, _VP, _VP, _VP, _VP, _VP, _VP, _VP]),
     "blr_scan_fwd_gated": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]),

@@ -270,8 +270,9 @@ blr_status seq_maps_gl(CUtensorMap* mr, CUtensorMap* mi, const void* base, const
 // z given: the merge of the gated layer is fused, and h receives y = h SiLU(z).
 blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const float* lambda,
                         const float* h0, void* h, float* h_last, unsigned char* w, cudaStream_t st,
-                        const void* z = nullptr) {
+                        const void* z, const int32_t* lengths) {
   blr::SeqFwdArgs a;
+  a.lengths = lengths;
   BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.sr));
   BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, plan.sr));
   a.write_h = h != nullptr;
@@ -303,8 +304,9 @@ blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const f
 blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, const void* x,
                         const void* gl, const float* lambda, const float* h0, void* dx, void* dgl,
                         float* dlambda, float* dh0, unsigned char* w, cudaStream_t st,
-                        const void* z = nullptr, void* dz = nullptr) {
+                        const void* z, void* dz, const int32_t* lengths) {
   blr::SeqBwdArgs a;
+  a.lengths = lengths;
   BLR_TRY(seq_maps_x(&a.tm_dh, dh, plan, plan.srb));
   BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.srb));
   BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, plan.srb));
@@ -354,13 +356,15 @@ blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fi
 // The tiled look-back kernels: a preparation kernel, then the scan.
 blr_status scan_fwd_tiled(const Plan& plan, const blr_desc* desc, const void* x,
                           const void* gate_logits, const float* lambda, const float* h0, void* h,
-                          float* h_last, unsigned char* w, cudaStream_t st) {
+                          float* h_last, unsigned char* w, cudaStream_t st,
+                          const int32_t* lengths) {
   // Clear the forward header (counters, error word), empty the
   // forward records, precompute k = -c softplus(Lambda).
   BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fpre,
                       plan.off_bagg - plan.off_fpre, reinterpret_cast<float*>(w + plan.off_k),
                       lambda, desc->D, desc->c, st));
   blr::FwdArgs a;
+  a.lengths = lengths;
   BLR_TRY(make_tensor_map(&a.tm_x, x, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
   BLR_TRY(make_tensor_map(&a.tm_gl, gate_logits, desc->io, 2 * desc->D, desc->L, desc->B, plan.tsteps));
   a.p = plan;
@@ -387,13 +391,15 @@ blr_status scan_fwd_tiled(const Plan& plan, const blr_desc* desc, const void* x,
 blr_status scan_bwd_tiled(const Plan& plan, const blr_desc* desc, const void* dh,
                           const float* dh_last, const void* x, const void* gate_logits,
                           const float* lambda, const float* h0, void* dx, void* dgate_logits,
-                          float* dlambda, float* dh0, unsigned char* w, cudaStream_t st) {
+                          float* dlambda, float* dh0, unsigned char* w, cudaStream_t st,
+                          const int32_t* lengths) {
   // Clear the backward header and the dLambda partial sums, empty the backward
   // records (the forward's records stay: they hold the carries).
   BLR_TRY(launch_prep(w + plan.off_bhdr, plan.off_k - plan.off_bhdr, w + plan.off_bagg,
                       plan.bytes - plan.off_bagg, reinterpret_cast<float*>(w + plan.off_k), lambda,
                       desc->D, desc->c, st));
   blr::BwdArgs a;
+  a.lengths = lengths;
   BLR_TRY(make_tensor_map(&a.tm_dh, dh, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
   BLR_TRY(make_tensor_map(&a.tm_x, x, desc->io, desc->D, desc->L, desc->B, plan.tsteps));
   BLR_TRY(make_tensor_map(&a.tm_gl, gate_logits, desc->io, 2 * desc->D, desc->L, desc->B, plan.tsteps));
@@ -463,7 +469,7 @@ blr_status launch_merge_bwd(int io, const void* dy, const void* z, void* dh, voi
 blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_logits,
                           const float* lambda, const float* h0, const void* z, void* h,
                           float* h_last, void* ws, size_t ws_bytes, blr_stream_t stream,
-                          bool gated) {
+                          bool gated, const int32_t* lengths = nullptr, bool varlen = false) {
   Plan plan;
   bool empty = false;
   BLR_TRY(check_desc(desc, &plan, &empty));
@@ -484,12 +490,14 @@ blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_
   BLR_TRY(need(gate_logits, "gate_logits", 16));
   BLR_TRY(optional(h, gated ? "y" : "h", 16));
   if (gated) BLR_TRY(need(z, "z", 16));
+  if (varlen) BLR_TRY(need(lengths, "lengths", 4));
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
   if (plan.seq)  // serial kernels (the merge fused): no preparation
-    return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st, h != nullptr ? z : nullptr);
-  BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, h, h_last, w, st));
+    return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st,
+                        h != nullptr ? z : nullptr, lengths);
+  BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, h, h_last, w, st, lengths));
   if (z == nullptr || h == nullptr) return BLR_OK;
   return launch_merge_fwd(desc->io, h, z, desc->B * desc->L * desc->D, st);
 }
@@ -499,7 +507,8 @@ blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_
 blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
                           const void* gate_logits, const float* lambda, const float* h0,
                           const void* z, void* dx, void* dgate_logits, void* dz, float* dlambda,
-                          float* dh0, void* ws, size_t ws_bytes, blr_stream_t stream, bool gated) {
+                          float* dh0, void* ws, size_t ws_bytes, blr_stream_t stream, bool gated,
+                          const int32_t* lengths = nullptr, bool varlen = false) {
   Plan plan;
   bool empty = false;
   BLR_TRY(check_desc(desc, &plan, &empty));
@@ -525,6 +534,7 @@ blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_
     BLR_TRY(need(z, "z", 16));
     BLR_TRY(need(dz, "dz", 16));
   }
+  if (varlen) BLR_TRY(need(lengths, "lengths", 4));
   BLR_TRY(need(x, "x", 16));
   BLR_TRY(need(gate_logits, "gate_logits", 16));
   BLR_TRY(need(dx, "dx", 16));
@@ -534,17 +544,17 @@ blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_
   unsigned char* w = static_cast<unsigned char*>(ws);
   if (plan.seq)  // the forward cleared the counters and partial sums
     return scan_bwd_seq(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
-                        dh0, w, st, z, dz);
+                        dh0, w, st, z, dz, lengths);
   if (z == nullptr)
     return scan_bwd_tiled(plan, desc, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
-                          dlambda, dh0, w, st);
+                          dlambda, dh0, w, st, lengths);
   // Gated, tiled: h recomputed into dz (a forward of the same problem, which
   // also rewrites the same carries), then dh = dy SiLU(z) into dx and
   // dz = dy h SiLU'(z), then the scan's backward from dh in dx.
-  BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, dz, nullptr, w, st));
+  BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, dz, nullptr, w, st, nullptr));
   BLR_TRY(launch_merge_bwd(desc->io, dh, z, dx, dz, desc->B * desc->L * desc->D, st));
   return scan_bwd_tiled(plan, desc, dx, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
-                        dlambda, dh0, w, st);
+                        dlambda, dh0, w, st, nullptr);
 }
 
 }  // namespace
@@ -569,6 +579,23 @@ blr_status blr_scan_fwd_gated(const blr_desc* desc, const void* x, const void* g
                               const float* lambda, const float* h0, const void* z, void* y,
                               float* h_last, void* ws, size_t ws_bytes, blr_stream_t stream) {
   return scan_fwd_entry(desc, x, gate_logits, lambda, h0, z, y, h_last, ws, ws_bytes, stream, true);
+}
+
+blr_status blr_scan_fwd_varlen(const blr_desc* desc, const int32_t* lengths, const void* x,
+                               const void* gate_logits, const float* lambda, const float* h0,
+                               void* h, float* h_last, void* ws, size_t ws_bytes,
+                               blr_stream_t stream) {
+  return scan_fwd_entry(desc, x, gate_logits, lambda, h0, nullptr, h, h_last, ws, ws_bytes, stream,
+                        false, lengths, true);
+}
+
+blr_status blr_scan_bwd_varlen(const blr_desc* desc, const int32_t* lengths, const void* dh,
+                               const float* dh_last, const void* x, const void* gate_logits,
+                               const float* lambda, const float* h0, void* dx, void* dgate_logits,
+                               float* dlambda, float* dh0, void* ws, size_t ws_bytes,
+                               blr_stream_t stream) {
+  return scan_bwd_entry(desc, dh, dh_last, x, gate_logits, lambda, h0, nullptr, dx, dgate_logits,
+                        nullptr, dlambda, dh0, ws, ws_bytes, stream, false, lengths, true);
 }
 
 blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,

@@ -30,6 +30,16 @@ namespace blr {
 
 constexpr unsigned kFull = 0xffffffffu;
 
+// The first step of row b's sequence: 0, or L - lengths[b] (lengths clamped to
+// [0, L]) when the rows carry their own lengths; the steps before it are
+// padding (Sec. 3.3's left padding), never read and never written.
+__device__ __forceinline__ int64_t row_start(const int32_t* lengths, int64_t b, int64_t L) {
+  if (lengths == nullptr) return 0;
+  int64_t n = lengths[b];
+  n = n < 0 ? 0 : (n > L ? L : n);
+  return L - n;
+}
+
 // Inputs reach the scan kernels through TMA tensor maps over 3-D views
 // (channels, time, batch) of the row-major tensors: x and dh as (D, L, B),
 // gate_logits as (2D, L, B).
@@ -37,6 +47,7 @@ struct FwdArgs {
   CUtensorMap tm_x;
   CUtensorMap tm_gl;
   Plan p;
+  const int32_t* lengths;  // NULL, or row b's sequence is its last lengths[b] steps
   const float* h0;
   void* h;
   float* h_last;
@@ -48,6 +59,7 @@ struct BwdArgs {
   CUtensorMap tm_x;
   CUtensorMap tm_gl;
   Plan p;
+  const int32_t* lengths;  // as FwdArgs
   const float* dh_last;
   const float* lambda;
   const float* h0;
@@ -302,12 +314,13 @@ __device__ __forceinline__ void lds_rows(const unsigned char* box, int row0, int
 
 // Forward gates of a lane's chunk: alpha and u = sqrt(1 - alpha^2) i x per
 // element; FULL when every element is inside the sequence and the channels,
-// else elements outside become the identity map (alpha = 1, u = 0).
+// else elements outside (rows before `lo` or from `valid` on) become the
+// identity map (alpha = 1, u = 0).
 template <class IO, class M, bool FULL>
 __device__ __forceinline__ void fwd_chunk(const float (&k)[4],
                                           const typename IO::Raw (&rx)[kTc],
                                           const typename IO::Raw (&rr)[kTc],
-                                          const typename IO::Raw (&ri)[kTc], int valid,
+                                          const typename IO::Raw (&ri)[kTc], int lo, int valid,
                                           float (&al)[kTc][4], float (&u)[kTc][4]) {
   float xv[kTc][4], rv[kTc][4], iv[kTc][4];
 #pragma unroll
@@ -341,7 +354,7 @@ __device__ __forceinline__ void fwd_chunk(const float (&k)[4],
   if (!FULL) {
 #pragma unroll
     for (int s = 0; s < kTc; ++s) {
-      if (s >= valid) {
+      if (s < lo || s >= valid) {
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
           al[s][v] = 1.0f;
@@ -425,7 +438,7 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
   TileCoord prev;
   prev.tile = p.n_tiles_f;  // none
   prev.tt = prev.cidx = prev.b = prev.dbase = 0;
-  int prev_valid = 0;
+  int prev_valid = 0, prev_lo = 0;
   float nk[VEC];
 #pragma unroll
   for (int v = 0; v < VEC; ++v) nk[v] = 0.0f;
@@ -445,11 +458,13 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
     if (!scanner) {
       // ---- consumers: tile it, gates and maps
       float al[kTc][VEC], u[kTc][VEC], ea[VEC], eu[VEC];
-      int valid = 0;
+      int valid = 0, lo = 0;
       if (cur_ok) {
         const int64_t d0 = tc.dbase + cv * VEC;
         const int64_t left = (d0 < p.D) ? p.L - (tc.tt * p.tsteps + row0) : 0;
         valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
+        const int64_t head = row_start(a.lengths, tc.b, p.L) - (tc.tt * p.tsteps + row0);
+        lo = (int)(head < 0 ? 0 : (head > kTc ? kTc : head));
         float k[VEC];
 #pragma unroll
         for (int v = 0; v < VEC; ++v) k[v] = nk[v];
@@ -467,10 +482,10 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
         lds_rows<IO>(sb, row0, cv, rx);
         lds_rows<IO>(sb + box_bytes<T>(), row0, cv, rr);
         lds_rows<IO>(sb + 2 * box_bytes<T>(), row0, cv, ri);
-        if (valid == kTc)
-          fwd_chunk<IO, M, true>(k, rx, rr, ri, valid, al, u);
+        if (valid == kTc && lo == 0)
+          fwd_chunk<IO, M, true>(k, rx, rr, ri, lo, valid, al, u);
         else
-          fwd_chunk<IO, M, false>(k, rx, rr, ri, valid, al, u);
+          fwd_chunk<IO, M, false>(k, rx, rr, ri, lo, valid, al, u);
         float A[VEC], U[VEC];
 #pragma unroll
         for (int v = 0; v < VEC; ++v) {
@@ -511,7 +526,7 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
       }
       __syncthreads();
       // ---- consumers: apply tile it-1 from the starting states the scanner wrote
-      if (prev_ok && h != nullptr && prev_valid > 0) {
+      if (prev_ok && h != nullptr && prev_valid > prev_lo) {
         const int64_t d0 = prev.dbase + cv * VEC;
         const int64_t t0 = prev.tt * p.tsteps + row0;
         float hs[VEC];
@@ -526,7 +541,7 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
             hs[v] = fmaf(pal[s][v], hs[v], pu[s][v]);
             out[v] = hs[v];
           }
-          if (s < prev_valid) IO::store(ph + s * p.D, out);
+          if (s >= prev_lo && s < prev_valid) IO::store(ph + s * p.D, out);
         }
       }
 #pragma unroll
@@ -542,6 +557,7 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
         peu[v] = eu[v];
       }
       prev_valid = valid;
+      prev_lo = lo;
     } else {
       // ---- scanner: tile it-1's carry and warp states, and the freed stage's
       // refill. The first look-back window is requested before anything else,
@@ -617,7 +633,7 @@ template <class IO, class M, bool FULL>
 __device__ __forceinline__ void bwd_chunk(const float (&k)[4], const typename IO::Raw (&rg)[kTc],
                                           const typename IO::Raw (&rx)[kTc],
                                           const typename IO::Raw (&rr)[kTc],
-                                          const typename IO::Raw (&ri)[kTc], int valid,
+                                          const typename IO::Raw (&ri)[kTc], int lo, int valid,
                                           float (&gv)[kTc][4], float (&xv)[kTc][4],
                                           float (&ev)[kTc][4], float (&rv)[kTc][4],
                                           float (&iv)[kTc][4], float (&A)[4], float (&U)[4],
@@ -659,7 +675,7 @@ __device__ __forceinline__ void bwd_chunk(const float (&k)[4], const typename IO
   if (!FULL) {
 #pragma unroll
     for (int s = 0; s < kTc; ++s) {
-      if (s >= valid) {
+      if (s < lo || s >= valid) {
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
           ev[s][v] = 0.0f;
@@ -772,6 +788,8 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
     const int64_t t0 = tc.tt * p.tsteps + row0;
     int64_t left = ch_ok ? p.L - t0 : 0;
     const int valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
+    const int64_t head = row_start(a.lengths, tc.b, p.L) - t0;
+    const int lo = (int)(head < 0 ? 0 : (head > kTc ? kTc : head));
     float k[VEC];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) k[v] = nk[v];
@@ -794,10 +812,10 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
       lds_rows<IO>(sb + box_bytes<T>(), row0, cv, rx);
       lds_rows<IO>(sb + 2 * box_bytes<T>(), row0, cv, rr);
       lds_rows<IO>(sb + 3 * box_bytes<T>(), row0, cv, ri);
-      if (valid == kTc)
-        bwd_chunk<IO, M, true>(k, rg, rx, rr, ri, valid, gv, xv, ev, rv, iv, A, U, W);
+      if (valid == kTc && lo == 0)
+        bwd_chunk<IO, M, true>(k, rg, rx, rr, ri, lo, valid, gv, xv, ev, rv, iv, A, U, W);
       else
-        bwd_chunk<IO, M, false>(k, rg, rx, rr, ri, valid, gv, xv, ev, rv, iv, A, U, W);
+        bwd_chunk<IO, M, false>(k, rg, rx, rr, ri, lo, valid, gv, xv, ev, rv, iv, A, U, W);
     }
     // 2. warp maps: h forwards (prefix), w backwards (suffix)
     float A2[VEC];
@@ -904,7 +922,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
         dlr[v] = fmaf(dl, r, dlr[v]);
         hs[v] = fmaf(alpha, hs[v], uu);
       }
-      if (s < valid) {
+      if (s >= lo && s < valid) {
         IO::store(pdx + s * p.D, ox);
         IO::store(pdg + s * 2 * p.D, orho);
         IO::store(pdg + s * 2 * p.D + p.D, oiota);

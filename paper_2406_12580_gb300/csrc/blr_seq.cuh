@@ -44,6 +44,7 @@ struct SeqFwdArgs {
   CUtensorMap tm_h;  // h, or y = h SiLU(z) when gated; unused when NULL
   CUtensorMap tm_z;  // gated: z, the merge gate's input
   Plan p;
+  const int32_t* lengths;  // NULL, or row b's sequence is its last lengths[b] steps
   const float* lambda;
   const float* h0;
   float* h_last;
@@ -63,6 +64,7 @@ struct SeqBwdArgs {
   CUtensorMap tm_z;   // gated: z
   CUtensorMap tm_dz;  // gated: dz
   Plan p;
+  const int32_t* lengths;  // as SeqFwdArgs
   const float* dh_last;
   const float* lambda;
   const float* h0;
@@ -232,11 +234,14 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
 #pragma unroll
   for (int v = 0; v < VEC; ++v) hc[v] = (ch_ok && a.h0 != nullptr) ? a.h0[b * p.D + d0 + v] : 0.0f;
 
-  const int64_t nblk = (p.L + R - 1) / R;
+  // The chain's steps: [t0, L) (all of them unless the rows carry lengths).
+  const int64_t t0 = row_start(a.lengths, b, p.L);
+  const int64_t len = p.L - t0;
+  const int64_t nblk = (len + R - 1) / R;
   const int cd = (int)(g * CHW), cb = (int)b;
   auto issue = [&](int st, int64_t j) {
     unsigned char* dst = ring.stage(st);
-    const int t = (int)(j * R);
+    const int t = (int)(t0 + j * R);
     mbar_arrive_expect_tx(&ring.bars[st], NB * BOX);
     tma_load_3d(dst, &a.tm_x, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + BOX, &a.tm_r, &ring.bars[st], cd, t, cb);
@@ -264,7 +269,7 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     }
     unsigned char* sb = ring.stage(st);
     unsigned char* lb = sb + lane * VEC * sizeof(T);
-    const int64_t left = p.L - j * R;
+    const int64_t left = len - j * R;
     const int rows = (int)(left < R ? left : R);
     if (rows == R) {
       if (poly)
@@ -277,7 +282,7 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     fence_proxy_async_smem();  // the stage's h rows, visible to the TMA store
     __syncwarp();
     if (lane == 0 && a.write_h) {
-      tma_store_3d(&a.tm_h, sb, cd, (int)(j * R), cb);
+      tma_store_3d(&a.tm_h, sb, cd, (int)(t0 + j * R), cb);
       bulk_commit();
     }
     prev = st;
@@ -467,11 +472,13 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     }
   };
 
-  const int64_t nblk = (p.L + R - 1) / R;
+  const int64_t t0 = row_start(a.lengths, b, p.L);
+  const int64_t len = p.L - t0;
+  const int64_t nblk = (len + R - 1) / R;
   const int cd = (int)(g * CHW), cb = (int)b;
   auto issue = [&](int st, int64_t j) {
     unsigned char* dst = ring.stage(st);
-    const int t = (int)(j * R);
+    const int t = (int)(t0 + j * R);
     mbar_arrive_expect_tx(&ring.bars[st], NB * BOX);
     tma_load_3d(dst, &a.tm_dh, &ring.bars[st], cd, t, cb);
     tma_load_3d(dst + BOX, &a.tm_x, &ring.bars[st], cd, t, cb);
@@ -486,7 +493,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   }
   __syncwarp();
 
-  int64_t m = (p.L + RB - 1) / RB - 1;  // the sub-block processed next
+  int64_t m = (len + RB - 1) / RB - 1;  // the sub-block processed next (-1: none)
 #pragma unroll
   for (int u = 0; u < QD; ++u) {
 #pragma unroll
@@ -505,7 +512,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     }
     unsigned char* sb = ring.stage(st);
     unsigned char* lb = sb + lane * VEC * sizeof(T);
-    const int64_t left = p.L - j * R;
+    const int64_t left = len - j * R;
     const int rows = (int)(left < R ? left : R);
 #pragma unroll
     for (int q = NSUB - 1; q >= 0; --q) {
@@ -535,7 +542,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     fence_proxy_async_smem();  // the stage's outputs, visible to the TMA stores
     __syncwarp();
     if (lane == 0) {
-      const int t = (int)(j * R);
+      const int t = (int)(t0 + j * R);
       tma_store_3d(&a.tm_dx, sb, cd, t, cb);
       tma_store_3d(&a.tm_dr, sb + 2 * BOX, cd, t, cb);
       tma_store_3d(&a.tm_di, sb + 3 * BOX, cd, t, cb);

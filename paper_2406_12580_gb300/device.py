@@ -11,8 +11,8 @@ from typing import Optional
 
 import numpy as np
 
-from . import (BLR_BF16, BLR_F32, Desc, blr_scan_bwd, blr_scan_bwd_gated, blr_scan_fwd,
-               blr_scan_fwd_gated, blr_step, blr_workspace_bytes)
+from . import (BLR_BF16, BLR_F32, Desc, blr_scan_bwd, blr_scan_bwd_gated, blr_scan_bwd_varlen,
+               blr_scan_fwd, blr_scan_fwd_gated, blr_scan_fwd_varlen, blr_step, blr_workspace_bytes)
 from .inputs import BF16, ScanInputs, StepInputs
 
 
@@ -97,6 +97,15 @@ class ScanBuffers:
     def bwd(self, stream=None):
         blr_scan_bwd(self.desc, self.dh, self.dh_last, self.x, self.gl, self.lam, self.h0, self.dx,
                      self.dgl, self.dlam, self.dh0, self.ws, stream)
+
+    def fwd_varlen(self, lengths, stream=None):
+        """The forward with per-row lengths (an int32 CUDA tensor of B)."""
+        blr_scan_fwd_varlen(self.desc, lengths, self.x, self.gl, self.lam, self.h0, self.h,
+                            self.h_last, self.ws, stream)
+
+    def bwd_varlen(self, lengths, stream=None):
+        blr_scan_bwd_varlen(self.desc, lengths, self.dh, self.dh_last, self.x, self.gl, self.lam,
+                            self.h0, self.dx, self.dgl, self.dlam, self.dh0, self.ws, stream)
 
     def fwd_gated(self, stream=None):
         """y = h SiLU(z) into self.h."""

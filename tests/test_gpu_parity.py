@@ -343,3 +343,50 @@ def test_steps(case, io, state):
     torch.cuda.synchronize()
     assert torch.equal(out, h)
     assert torch.equal(h2, out)
+
+
+# Rows of their own lengths (blr_scan_*_varlen): sequences right-aligned in
+# their rows (left padding), padding never read or written; both kernel
+# families, empty and full rows included.
+VARLEN = [dict(B=3, L=65, D=72, random_h0=True, random_dh_last=True),
+          dict(B=2, L=300, D=16),
+          dict(B=300, L=203, D=24, random_h0=True, random_dh_last=True),
+          dict(B=700, L=37, D=40, decay=(0.05, 0.95), c=2.0),
+          dict(B=260, L=1100, D=8, decay=(0.99, 0.9999), random_h0=True)]
+
+
+@pytest.mark.parametrize("io", [I.F32, I.BF16])
+@pytest.mark.parametrize("case", range(len(VARLEN)))
+def test_varlen(io, case):
+    import oracle
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = _cfg(io, 600 + case, **VARLEN[case])
+    inp = I.make_scan_inputs(cfg)
+    B, L, D = cfg.B, cfg.L, cfg.D
+    lengths = np.random.default_rng(case).integers(0, L + 1, size=B).astype(np.int32)
+    lengths[0] = L
+    lengths[1] = 0
+    lengths[-1] = min(L, 3)
+    buf = ScanBuffers.from_inputs(inp)
+    for t in (buf.h, buf.dx, buf.dgl):
+        t.fill_(float("nan"))
+    lt = torch.from_numpy(lengths).cuda()
+    buf.fwd_varlen(lt)
+    buf.bwd_varlen(lt)
+    torch.cuda.synchronize()
+    orc = oracle.load()
+    h, h_last = orc.fwd_varlen(lengths, inp.x, inp.gl, inp.lam, inp.h0, c=cfg.c)
+    dx, dgl, dlam, dh0 = orc.bwd_varlen(lengths, inp.dh, inp.x, inp.gl, inp.lam, inp.h0,
+                                        inp.dh_last, c=cfg.c)
+    got = gpu_outputs(buf)
+    real = ~np.isnan(h)
+    real2 = np.concatenate([real, real], axis=2)
+    tol = TOL[io]
+    # the padding keeps what the caller left there: nothing was written
+    assert np.isnan(got["h"][~real]).all() and np.isnan(got["dx"][~real]).all()
+    assert np.isnan(got["dgl"][~real2]).all()
+    assert normwise(got["h"][real], h[real]) <= tol
+    assert normwise(got["dx"][real], dx[real]) <= tol
+    assert normwise(got["dgl"][real2], dgl[real2]) <= tol
+    for k, w in (("h_last", h_last), ("dlam", dlam), ("dh0", dh0)):
+        assert normwise(got[k], w) <= tol, k
