@@ -532,6 +532,8 @@ def other_workloads(flush, peak, dev, headline):
     for k in (1, 2):
         out[f"gated_config{k}"] = gated_workload(k, flush, peak, dev)
     out["gated_layer_train_step"] = layer_workload(flush, dev)
+    out["varlen_config2"] = varlen_workload(flush, peak, dev)
+    out["padding_table"] = padding_table(flush, dev)
     return out
 
 
@@ -565,6 +567,61 @@ def steps_workload(io, flush, peak, dev, B=65536, K=8, D=64, reps=20):
     gbs = B * D * (2 + 3 * K) * ib / (ms * 1e-3) / 1e9
     return {"workload": cfg.name + " in one call", "ms": ms,
             "steps_per_s": B * D * K / (ms * 1e-3), "gbs": gbs, "frac": gbs / peak}
+
+
+def _time_fwd_bwd(fwd, bwd, flush, reps):
+    import torch
+    for _ in range(3):
+        fwd(); bwd()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
+    for e in ev:
+        flush()
+        e[0].record(); fwd(); e[1].record(); bwd(); e[2].record()
+    torch.cuda.synchronize()
+    return (statistics.median(a.elapsed_time(b) for a, b, c in ev),
+            statistics.median(b.elapsed_time(c) for a, b, c in ev))
+
+
+def varlen_workload(flush, peak, dev, reps=20):
+    """The train-shaped workload (20 % of every row left padding) given as rows
+    of their own length, 40 of 50 steps (blr_scan_*_varlen: the padding is not
+    read), against the padded scan over all 50."""
+    import torch
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = I.CONFIGS[2]
+    buf = ScanBuffers.from_inputs(I.make_scan_inputs(cfg), device=dev)
+    lengths = torch.full((cfg.B,), cfg.L - cfg.pad_rows, dtype=torch.int32, device=dev)
+    fp, bp = _time_fwd_bwd(buf.fwd, buf.bwd, flush, reps)
+    fv, bv = _time_fwd_bwd(lambda: buf.fwd_varlen(lengths), lambda: buf.bwd_varlen(lengths),
+                           flush, reps)
+    n_real = cfg.B * (cfg.L - cfg.pad_rows) * cfg.D
+    gbs = n_real * 22 * io_bytes(cfg.io) / 2 / ((fv + bv) * 1e-3) / 1e9
+    return {"workload": cfg.name + f", as rows of {cfg.L - cfg.pad_rows} steps",
+            "padded": {"fwd_ms": fp, "bwd_ms": bp}, "varlen": {"fwd_ms": fv, "bwd_ms": bv},
+            "speedup": (fp + bp) / (fv + bv), "varlen_gbs": gbs, "varlen_frac": gbs / peak}
+
+
+def padding_table(flush, dev, B=256, D=64, reps=20):
+    """The shape of the paper's padding comparison (Sec. 4, lengths 200, 100,
+    257): fwd + bwd of the sequence length itself (this scan needs no padding)
+    against the same scan over the next power of two, the length a two-tree
+    scan needs."""
+    from paper_2406_12580_gb300 import inputs as I
+    from paper_2406_12580_gb300.device import ScanBuffers
+    rows = {}
+    for L in (200, 100, 257):
+        L2 = 1 << (L - 1).bit_length()
+        t = {}
+        for n in (L, L2):
+            cfg = I.ScanConfig(f"fwd+bwd B={B} L={n} D={D} fp32", B, n, D, "f32", seed=5)
+            buf = ScanBuffers.from_inputs(I.make_scan_inputs(cfg), device=dev)
+            f, b = _time_fwd_bwd(buf.fwd, buf.bwd, flush, reps)
+            t[n] = f + b
+            del buf
+        rows[f"L={L}"] = {"ms": t[L], f"ms_at_L={L2}": t[L2], "padded_over_exact": t[L2] / t[L]}
+    return {"workload": f"fwd+bwd B={B} D={D} fp32 at L and at the next power of two",
+            "rows": rows}
 
 
 def layer_workload(flush, dev, B=256, L=200, D=64, E=2, reps=10):
