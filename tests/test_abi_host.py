@@ -192,3 +192,14 @@ def test_status_strings(lib):
         s = lib.blr_status_string(code)
         assert s and s.startswith(b"BLR_")
     assert b"unknown" in lib.blr_status_string(99)
+
+
+def test_no_library_no_fallback(monkeypatch, tmp_path):
+    """Without libblr.so every entry point raises: there is no CPU path."""
+    import paper_2406_12580_gb300 as P
+    monkeypatch.setattr(_lib, "_lib", None)
+    monkeypatch.setattr(_lib, "library_path", lambda: str(tmp_path / "libblr.so"))
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        P.blr_workspace_bytes(D(2, 4, 8))
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        P.blr_status_string(0)
