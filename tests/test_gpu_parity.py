@@ -390,3 +390,85 @@ def test_varlen(io, case):
     assert normwise(got["dgl"][real2], dgl[real2]) <= tol
     for k, w in (("h_last", h_last), ("dlam", dlam), ("dh0", dh0)):
         assert normwise(got[k], w) <= tol, k
+
+
+# Seeded random problems across the whole surface: dtype, shape, h0 / dh_last,
+# c, decays, row lengths and the gated merge drawn at random (fixed seeds).
+def _fuzz_case(seed):
+    rng = np.random.default_rng(seed)
+    io = [I.F32, I.BF16][rng.integers(2)]
+    B = int(rng.choice([1, 2, 5, 40, 300, 700]))
+    D = int(8 * rng.integers(1, 17))
+    L = int(rng.integers(1, max(2, min(400, 1_000_000 // (B * D)))))  # the oracle stays quick
+    lo = float(rng.choice([0.05, 0.5, 0.9, 0.99]))
+    kw = dict(B=B, L=L, D=D, decay=(lo, min(0.9999, lo + 0.09)), c=float(rng.choice([0.5, 1.0, 3.0])),
+              random_h0=bool(rng.integers(2)), random_dh_last=bool(rng.integers(2)),
+              gate_std=float(rng.choice([0.5, 1.0, 3.0])))
+    mode = ["plain", "gated", "varlen"][rng.integers(3)]
+    return io, kw, mode, rng
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_fuzz(seed):
+    import oracle
+    io, kw, mode, rng = _fuzz_case(seed)
+    cfg = _cfg(io, 700 + seed, gated=(mode == "gated"), **kw)
+    inp = I.make_scan_inputs(cfg)
+    if mode == "gated":
+        compare(inp, gpu_outputs(gpu_scan_gated(inp)), oracle_outputs(inp))
+    elif mode == "plain":
+        compare(inp, gpu_outputs(gpu_scan(inp)), oracle_outputs(inp))
+    else:
+        from paper_2406_12580_gb300.device import ScanBuffers
+        lengths = rng.integers(0, cfg.L + 1, size=cfg.B).astype(np.int32)
+        buf = ScanBuffers.from_inputs(inp)
+        for t in (buf.h, buf.dx, buf.dgl):
+            t.zero_()  # the padding is not written: keep it defined
+        lt = torch.from_numpy(lengths).cuda()
+        buf.fwd_varlen(lt)
+        buf.bwd_varlen(lt)
+        torch.cuda.synchronize()
+        orc = oracle.load()
+        h, h_last = orc.fwd_varlen(lengths, inp.x, inp.gl, inp.lam, inp.h0, c=cfg.c)
+        dx, dgl, dlam, dh0 = orc.bwd_varlen(lengths, inp.dh, inp.x, inp.gl, inp.lam, inp.h0,
+                                            inp.dh_last, c=cfg.c)
+        got = gpu_outputs(buf)
+        real = ~np.isnan(h)
+        real2 = np.concatenate([real, real], axis=2)
+        tol = TOL[io]
+        assert normwise(got["h"][real], h[real]) <= tol
+        assert normwise(got["dx"][real], dx[real]) <= tol
+        assert normwise(got["dgl"][real2], dgl[real2]) <= tol
+        for k, w in (("h_last", h_last), ("dlam", dlam), ("dh0", dh0)):
+            assert normwise(got[k], w) <= tol, k
+
+
+@pytest.mark.parametrize("shape", [dict(B=300, L=130, D=40), dict(B=3, L=300, D=72)])
+def test_graph_capture_replays_eager(shape):
+    """The forward and backward captured into a CUDA graph (no host work is
+    needed between them) replay to the eager results, on both kernel families."""
+    inp = I.make_scan_inputs(_cfg(I.F32, 900, random_h0=True, random_dh_last=True, **shape))
+    eager = gpu_outputs(gpu_scan(inp))
+    from paper_2406_12580_gb300.device import ScanBuffers
+    buf = ScanBuffers.from_inputs(inp)
+    buf.fwd()
+    buf.bwd()  # first calls outside capture (per-device setup)
+    torch.cuda.synchronize()
+    for t in (buf.h, buf.dx, buf.dgl, buf.dlam):
+        t.zero_()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(g, stream=side):
+            buf.fwd()
+            buf.bwd()
+    torch.cuda.current_stream().wait_stream(side)
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    got = gpu_outputs(buf)
+    # the same kernels, so the same values up to the order of float atomics
+    # (dLambda) and of look-back combines (the tiled kernels)
+    for k in eager:
+        assert normwise(got[k], eager[k]) <= 1e-6, k
