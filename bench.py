@@ -206,13 +206,13 @@ class ClockSampler:
 
 # ------------------------------------------------------------ CPU baseline
 
-def cpu_oracle_rate(inp, target_s: float = 10.0, max_reps: int = 50):
-    """The float64 oracle, as it stands, on the host cores: fwd + bwd over the
-    whole workload, repeated for about `target_s` seconds. Returns
-    (elements/s, threads, reps, seconds)."""
+def cpu_oracle_rate(inp, target_s: float = 10.0, max_reps: int = 1000, threads: int = 0):
+    """The float64 oracle, as it stands, on the host cores (all of them, or
+    `threads`): fwd + bwd over the whole workload, repeated for about
+    `target_s` seconds. Returns (elements/s, threads, reps, seconds)."""
     import oracle
     orc = oracle.load()
-    threads = os.cpu_count() or 1
+    threads = threads or os.cpu_count() or 1
     n = inp.cfg.elements
     t = time.perf_counter()
     reps = 0
@@ -455,9 +455,12 @@ def run_ours(args):
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rate, threads, reps, secs = cpu_oracle_rate(inp)
+        rate1, _, reps1, secs1 = cpu_oracle_rate(inp, target_s=3.0, threads=1)
         line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                                 "sample": f"{reps} x fwd+bwd of the whole workload "
-                                          f"({n} elements) in {secs:.1f} s, float64"}
+                                          f"({n} elements) in {secs:.1f} s, float64",
+                                "single_thread": {"value": rate1, "unit": UNIT, "cores": 1,
+                                                  "sample": f"{reps1} x fwd+bwd in {secs1:.1f} s"}}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
