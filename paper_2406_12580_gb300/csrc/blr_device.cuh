@@ -77,6 +77,13 @@ struct Io<__nv_bfloat16, 4> {  // 8 bytes
   static __device__ __forceinline__ void store(T* p, const float (&v)[4]) {
     __stcs(reinterpret_cast<uint2*>(p), make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3])));
   }
+  // v = t / 2, halved on the packed pairs (an exponent decrement).
+  static __device__ __forceinline__ void unpack_half(const Raw& t, float (&v)[4]) {
+    uint32_t a, b;
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(t.x), "r"(0x3f003f00u));
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(b) : "r"(t.y), "r"(0x3f003f00u));
+    v[0] = bf16_lo(a); v[1] = bf16_hi(a); v[2] = bf16_lo(b); v[3] = bf16_hi(b);
+  }
 };
 
 template <>

@@ -323,22 +323,45 @@ __device__ __forceinline__ void fwd_chunk(const float (&k)[4],
                                           const typename IO::Raw (&ri)[kTc], int lo, int valid,
                                           float (&al)[kTc][4], float (&u)[kTc][4]) {
   float xv[kTc][4], rv[kTc][4], iv[kTc][4];
+  using G = typename GatePolicy<M>::type;
+  constexpr bool HALF = G::kHalfInputs && sizeof(typename IO::T) == 2;
 #pragma unroll
   for (int s = 0; s < kTc; ++s) {
-    IO::unpack(rx[s], xv[s]);
-    IO::unpack(rr[s], rv[s]);
-    IO::unpack(ri[s], iv[s]);
+    if constexpr (HALF) {
+      IO::unpack_half(rx[s], xv[s]);
+      IO::unpack_half(rr[s], rv[s]);
+      IO::unpack_half(ri[s], iv[s]);
+    } else {
+      IO::unpack(rx[s], xv[s]);
+      IO::unpack(rr[s], rv[s]);
+      IO::unpack(ri[s], iv[s]);
+    }
   }
 #pragma unroll
   for (int v = 0; v < 4; ++v) {
     if (k[v] >= -kPolyLimit) {
+      const float kh = 0.5f * k[v];
 #pragma unroll
       for (int s = 0; s < kTc; ++s) {
-        const float r = M::sigmoid(rv[s][v]);
-        const float i = M::sigmoid(iv[s][v]);
-        const float e = gate_expm1<M, true>(k[v] * r);
+        if constexpr (HALF) {
+          const float e = gate_expm1<M, true>(G::decay_log_half(rv[s][v], kh));
+          al[s][v] = 1.0f + e;
+          u[s][v] = M::sqrt(-e * (2.0f + e)) * G::gated_x_half(iv[s][v], xv[s][v]);
+        } else {
+          const float r = M::sigmoid(rv[s][v]);
+          const float i = M::sigmoid(iv[s][v]);
+          const float e = gate_expm1<M, true>(k[v] * r);
+          al[s][v] = 1.0f + e;
+          u[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
+        }
+      }
+    } else if constexpr (HALF) {
+      const float kh = 0.5f * k[v];
+#pragma unroll
+      for (int s = 0; s < kTc; ++s) {
+        const float e = gate_expm1<M, false>(G::decay_log_half(rv[s][v], kh));
         al[s][v] = 1.0f + e;
-        u[s][v] = M::sqrt(-e * (2.0f + e)) * i * xv[s][v];
+        u[s][v] = M::sqrt(-e * (2.0f + e)) * G::gated_x_half(iv[s][v], xv[s][v]);
       }
     } else {
 #pragma unroll
