@@ -232,9 +232,9 @@ blr_status allow_smem(K kernel, size_t smem) {
                     "set dynamic shared memory size");
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED>
+template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN = false>
 blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED>;
+  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED, VARLEN>;
   constexpr int NB = GATED ? 4 : 3;
   a.stages = seq_stages(a.p.n_chain, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
   const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
@@ -243,9 +243,9 @@ blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
   return cuda_check(cudaGetLastError(), "launch seq_fwd_kernel");
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED>
+template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN = false>
 blr_status launch_seq_bwd(blr::SeqBwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED>;
+  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED, VARLEN>;
   constexpr int NB = GATED ? 5 : 4;
   a.stages = seq_stages(a.p.n_chain, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
   const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
@@ -293,6 +293,13 @@ blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const f
     }
     return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, true>(a, st);
   }
+  if (lengths != nullptr) {
+    if (plan.io == BLR_F32) {
+      if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, false, true>(a, st);
+      return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16, false, true>(a, st);
+    }
+    return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, false, true>(a, st);
+  }
   if (plan.io == BLR_F32) {
     if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, false>(a, st);
     return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16, false>(a, st);
@@ -332,6 +339,10 @@ blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, 
     if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, true>(a, st);
     return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, true>(a, st);
   }
+  if (lengths != nullptr) {
+    if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, false, true>(a, st);
+    return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false, true>(a, st);
+  }
   if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, false>(a, st);
   return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false>(a, st);
 }
@@ -353,6 +364,26 @@ blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fi
   return cuda_check(cudaGetLastError(), "launch prep_kernel");
 }
 
+template <typename T, class M, bool VARLEN>
+blr_status launch_tiled_fwd(const Plan& plan, const blr::FwdArgs& a, cudaStream_t st) {
+  const int threads = (plan.nwarps + 1) * 32;  // consumer warps + the scanner warp
+  auto k = blr::scan_fwd_kernel<T, M, VARLEN>;
+  const size_t smem = blr::ring_bytes<T, blr::fwd_stages<T>(), 3>();
+  unsigned grid = 1;
+  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
+  return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel");
+}
+
+template <typename T, class M, bool VARLEN>
+blr_status launch_tiled_bwd(const Plan& plan, const blr::BwdArgs& a, cudaStream_t st) {
+  const int threads = plan.nwarps * 32;
+  auto k = blr::scan_bwd_kernel<T, M, VARLEN>;
+  const size_t smem = blr::ring_bytes<T, blr::bwd_stages<T>(), 4>();
+  unsigned grid = 1;
+  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
+  return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel");
+}
+
 // The tiled look-back kernels: a preparation kernel, then the scan.
 blr_status scan_fwd_tiled(const Plan& plan, const blr_desc* desc, const void* x,
                           const void* gate_logits, const float* lambda, const float* h0, void* h,
@@ -372,18 +403,12 @@ blr_status scan_fwd_tiled(const Plan& plan, const blr_desc* desc, const void* x,
   a.h = h;
   a.h_last = h_last;
   a.ws = w;
-  const int threads = (plan.nwarps + 1) * 32;  // consumer warps + the scanner warp
-  unsigned grid = 1;
   if (desc->io == BLR_F32) {
-    auto k = blr::scan_fwd_kernel<float, blr::MathPrecise>;
-    const size_t smem = blr::ring_bytes<float, blr::fwd_stages<float>(), 3>();
-    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
-    return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel");
+    if (lengths != nullptr) return launch_tiled_fwd<float, blr::MathPrecise, true>(plan, a, st);
+    return launch_tiled_fwd<float, blr::MathPrecise, false>(plan, a, st);
   }
-  auto k = blr::scan_fwd_kernel<__nv_bfloat16, blr::MathFast>;
-  const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::fwd_stages<__nv_bfloat16>(), 3>();
-  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_f, &grid));
-  return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_fwd_kernel");
+  if (lengths != nullptr) return launch_tiled_fwd<__nv_bfloat16, blr::MathFast, true>(plan, a, st);
+  return launch_tiled_fwd<__nv_bfloat16, blr::MathFast, false>(plan, a, st);
 }
 
 // dh may be the dx buffer itself: every element of dh is read (into shared
@@ -412,18 +437,12 @@ blr_status scan_bwd_tiled(const Plan& plan, const blr_desc* desc, const void* dh
   a.dlambda = dlambda;
   a.dh0 = dh0;
   a.ws = w;
-  const int threads = plan.nwarps * 32;
-  unsigned grid = 1;
   if (desc->io == BLR_F32) {
-    auto k = blr::scan_bwd_kernel<float, blr::MathPrecise>;
-    const size_t smem = blr::ring_bytes<float, blr::bwd_stages<float>(), 4>();
-    BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
-    return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel");
+    if (lengths != nullptr) return launch_tiled_bwd<float, blr::MathPrecise, true>(plan, a, st);
+    return launch_tiled_bwd<float, blr::MathPrecise, false>(plan, a, st);
   }
-  auto k = blr::scan_bwd_kernel<__nv_bfloat16, blr::MathFast>;
-  const size_t smem = blr::ring_bytes<__nv_bfloat16, blr::bwd_stages<__nv_bfloat16>(), 4>();
-  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tiles_b, &grid));
-  return launch_cooperative(k, grid, threads, smem, st, a, "launch scan_bwd_kernel");
+  if (lengths != nullptr) return launch_tiled_bwd<__nv_bfloat16, blr::MathFast, true>(plan, a, st);
+  return launch_tiled_bwd<__nv_bfloat16, blr::MathFast, false>(plan, a, st);
 }
 
 // Grid of the elementwise merge kernels: 16-byte vectors, 256 threads a block,

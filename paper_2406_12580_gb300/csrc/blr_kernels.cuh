@@ -399,7 +399,9 @@ __device__ __forceinline__ void fwd_chunk(const float (&k)[4],
 // they kept in registers). The scanner's round trips to L2 thus overlap the
 // consumers' arithmetic.
 
-template <typename T, class M>
+// VARLEN: the rows carry lengths (a.lengths), whose padding the kernel masks;
+// the form without keeps the registers of the plain scan.
+template <typename T, class M, bool VARLEN>
 __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
     scan_fwd_kernel(const __grid_constant__ FwdArgs a) {
   using IO = Io<T, 4>;
@@ -486,8 +488,10 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
         const int64_t d0 = tc.dbase + cv * VEC;
         const int64_t left = (d0 < p.D) ? p.L - (tc.tt * p.tsteps + row0) : 0;
         valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
-        const int64_t head = row_start(a.lengths, tc.b, p.L) - (tc.tt * p.tsteps + row0);
-        lo = (int)(head < 0 ? 0 : (head > kTc ? kTc : head));
+        if constexpr (VARLEN) {
+          const int64_t head = row_start(a.lengths, tc.b, p.L) - (tc.tt * p.tsteps + row0);
+          lo = (int)(head < 0 ? 0 : (head > kTc ? kTc : head));
+        }
         float k[VEC];
 #pragma unroll
         for (int v = 0; v < VEC; ++v) k[v] = nk[v];
@@ -580,7 +584,7 @@ __global__ void __launch_bounds__((kMaxWarps + 1) * 32, sizeof(T) == 4 ? 2 : 3)
         peu[v] = eu[v];
       }
       prev_valid = valid;
-      prev_lo = lo;
+      if constexpr (VARLEN) prev_lo = lo;
     } else {
       // ---- scanner: tile it-1's carry and warp states, and the freed stage's
       // refill. The first look-back window is requested before anything else,
@@ -726,7 +730,7 @@ __device__ __forceinline__ void bwd_chunk(const float (&k)[4], const typename IO
   }
 }
 
-template <typename T, class M>
+template <typename T, class M, bool VARLEN>
 __global__ void __launch_bounds__(kMaxWarps * 32, 3)
     scan_bwd_kernel(const __grid_constant__ BwdArgs a) {
   using IO = Io<T, 4>;
@@ -811,8 +815,11 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
     const int64_t t0 = tc.tt * p.tsteps + row0;
     int64_t left = ch_ok ? p.L - t0 : 0;
     const int valid = (int)(left < 0 ? 0 : (left > kTc ? kTc : left));
-    const int64_t head = row_start(a.lengths, tc.b, p.L) - t0;
-    const int lo = (int)(head < 0 ? 0 : (head > kTc ? kTc : head));
+    int lo = 0;
+    if constexpr (VARLEN) {
+      const int64_t head = row_start(a.lengths, tc.b, p.L) - t0;
+      lo = (int)(head < 0 ? 0 : (head > kTc ? kTc : head));
+    }
     float k[VEC];
 #pragma unroll
     for (int v = 0; v < VEC; ++v) k[v] = nk[v];

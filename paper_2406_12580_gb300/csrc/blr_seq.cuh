@@ -195,7 +195,9 @@ __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
   }
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED>
+// VARLEN: the rows carry lengths (a.lengths) and each chain starts at its
+// first real step; the form without keeps the plain scan's code.
+template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN>
 __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ SeqFwdArgs a) {
   using IO = Io<T, VEC>;
   using G = typename GatePolicy<M>::type;
@@ -235,7 +237,7 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
   for (int v = 0; v < VEC; ++v) hc[v] = (ch_ok && a.h0 != nullptr) ? a.h0[b * p.D + d0 + v] : 0.0f;
 
   // The chain's steps: [t0, L) (all of them unless the rows carry lengths).
-  const int64_t t0 = row_start(a.lengths, b, p.L);
+  const int64_t t0 = VARLEN ? row_start(a.lengths, b, p.L) : 0;
   const int64_t len = p.L - t0;
   const int64_t nblk = (len + R - 1) / R;
   const int cd = (int)(g * CHW), cb = (int)b;
@@ -415,7 +417,7 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
   }
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED>
+template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN>
 __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(const __grid_constant__ SeqBwdArgs a) {
   using IO = Io<T, VEC>;
   using G = typename GatePolicy<M>::type;
@@ -472,7 +474,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     }
   };
 
-  const int64_t t0 = row_start(a.lengths, b, p.L);
+  const int64_t t0 = VARLEN ? row_start(a.lengths, b, p.L) : 0;
   const int64_t len = p.L - t0;
   const int64_t nblk = (len + R - 1) / R;
   const int cd = (int)(g * CHW), cb = (int)b;
