@@ -89,12 +89,15 @@ typedef struct {
 } blr_desc;
 
 /*
- * Workspace size in bytes for blr_scan_fwd / blr_scan_bwd on `desc`; 0 when
- * the description is invalid or needs none (B, L or D zero). The workspace
- * holds per-tile carries of the forward (reused by the backward), per-tile
- * state of the inter-block scans, and the float64 partial sums of dlambda:
- * about 24 bytes per channel per tile of up to 64 time steps (under 0.4
- * bytes per element), plus 64 bytes per channel. It depends only on B, L, D.
+ * Workspace size in bytes for blr_scan_fwd / blr_scan_bwd (and their _gated
+ * and _varlen forms) on `desc`; 0 when the description is invalid or needs none
+ * (B, L or D zero). The workspace holds the states the forward keeps for the
+ * backward (every 16 float32 / 8 bfloat16 steps when the problem has at least
+ * 256 chains of 32 float32 or 64 bfloat16 channels: 0.25-0.5 bytes per
+ * element), or else the per-tile records of the tiled scans (24 bytes per
+ * channel per 64-step tile, under 0.4 bytes per element), plus the float64
+ * partial sums of dlambda and a small header (about 72 bytes per channel). It
+ * depends only on B, L, D and the I/O dtype.
  */
 BLR_API size_t blr_workspace_bytes(const blr_desc* desc);
 
@@ -112,7 +115,7 @@ BLR_API size_t blr_workspace_bytes(const blr_desc* desc);
  * ws, ws_bytes           device workspace of at least blr_workspace_bytes(desc)
  *                        bytes, 16-byte aligned. Its previous contents are
  *                        ignored; on return (in stream order) it holds the
- *                        per-tile carries that blr_scan_bwd consumes.
+ *                        kept states that blr_scan_bwd consumes.
  */
 BLR_API blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_logits,
                         const float* lambda, const float* h0, void* h, float* h_last, void* ws,
@@ -139,7 +142,7 @@ BLR_API blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void*
  *             carries of a completed forward of the same desc, no output is
  *             written and blr_workspace_status() reports BLR_ERR_WORKSPACE. The
  *             forward's carries survive the call, so the backward may be repeated.
- * h_{t-1} is recomputed from the forward's per-tile carries, not read from h.
+ * h_{t-1} is recomputed from the forward's kept states, not read from h.
  */
 BLR_API blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
                         const void* gate_logits, const float* lambda, const float* h0, void* dx,
