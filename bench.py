@@ -119,16 +119,18 @@ def kernel_sources_sha() -> str:
 
 
 def scan_kernels(cfg):
-    """(forward kernel, backward kernel, launches per call) of the family the
-    library picks for this shape: the serial kernels when there are at least
-    256 chains of 32 float32 or 64 bfloat16 channels, one launch per call;
-    otherwise the tiled look-back kernels, each after its preparation kernel.
-    (Mirrors the library's plan; used for labels and launch counts only.)"""
-    per_lane = 1 if cfg.io == "f32" else 2
-    chains = cfg.B * -(-cfg.D // (32 * per_lane))
-    if chains >= 256:
-        return "seq_fwd_kernel", "seq_bwd_kernel", 1
-    return "scan_fwd_kernel", "scan_bwd_kernel", 2
+    """(forward kernels, backward kernels, launches per call, what a call's
+    CUDA events bracket) of the family the library runs on this shape
+    (blr_scan_family)."""
+    from paper_2406_12580_gb300 import (FAMILY_SEGMENTED, FAMILY_SERIAL, Desc,
+                                        blr_scan_family)
+    fam = blr_scan_family(Desc(cfg.B, cfg.L, cfg.D, 0 if cfg.io == "f32" else 1, cfg.c))
+    if fam == FAMILY_SERIAL:
+        return "seq_fwd_kernel", "seq_bwd_kernel", 1, "the kernel alone"
+    if fam == FAMILY_SEGMENTED:
+        return ("seg_reduce_kernel+seq_fwd_kernel", "seg_reduce_kernel+seq_bwd_kernel", 2,
+                "the segment reduction and the serial kernel")
+    return "scan_fwd_kernel", "scan_bwd_kernel", 2, "the kernel and its preparation kernel"
 
 
 def ncu_traffic(kernel: str, workload: str):
@@ -410,14 +412,13 @@ def run_ours(args):
     favg = sum(fwd_ms) / len(fwd_ms)
     bavg = sum(bwd_ms) / len(bwd_ms) if bwd_ms and not cfg.fwd_only else 0.0
     ib = io_bytes(cfg.io)
-    fwd_kernel, bwd_kernel, per_call = scan_kernels(cfg)
+    fwd_kernel, bwd_kernel, per_call, bracket = scan_kernels(cfg)
     if bavg > favg:
         kname, avg_ms, alg = bwd_kernel, bavg, n * BWD_VALUES * ib
     else:
         kname, avg_ms, alg = fwd_kernel, favg, n * FWD_VALUES * ib
     achieved = alg / (avg_ms * 1e-3) / 1e9
-    timing = ("CUDA events around each C-ABI call (the kernel alone)" if per_call == 1 else
-              "CUDA events around each C-ABI call (the kernel and its preparation kernel)")
+    timing = f"CUDA events around each C-ABI call ({bracket})"
     roofline = {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
                 "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": ncu_traffic(kname, f"config{args.config}"),

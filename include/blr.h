@@ -91,15 +91,44 @@ typedef struct {
 /*
  * Workspace size in bytes for blr_scan_fwd / blr_scan_bwd (and their _gated
  * and _varlen forms) on `desc`; 0 when the description is invalid or needs none
- * (B, L or D zero). The workspace holds the states the forward keeps for the
- * backward (every 16 float32 / 8 bfloat16 steps when the problem has at least
- * 256 chains of 32 float32 or 64 bfloat16 channels: 0.25-0.5 bytes per
- * element), or else the per-tile records of the tiled scans (24 bytes per
- * channel per 64-step tile, under 0.4 bytes per element), plus the float64
- * partial sums of dlambda and a small header (about 72 bytes per channel). It
- * depends only on B, L, D and the I/O dtype.
+ * (B, L or D zero). The workspace holds what the forward keeps for the
+ * backward, by kernel family (blr_scan_family):
+ *   serial: the state every 16 float32 / 8 bfloat16 steps, 0.25-0.5 bytes per
+ *           element;
+ *   tiled: per-tile records (24 bytes per channel per 64-step tile, under 0.4
+ *           bytes per element);
+ *   segmented: the serial kernels' kept states and 12 bytes per channel per
+ *           segment (of 128 steps or more), laid over the tiled forward
+ *           records, plus the tiled backward records (for the _varlen forms),
+ *           under 0.8 bytes per element;
+ * plus the float64 partial sums of dlambda and a small header (about 72 bytes
+ * per channel). It depends only on B, L, D and the I/O dtype.
  */
 BLR_API size_t blr_workspace_bytes(const blr_desc* desc);
+
+/*
+ * Which kernels blr_scan_fwd / blr_scan_bwd (and their _gated forms; the
+ * _varlen forms when with_lengths is nonzero) run on `desc` (diagnostic; the
+ * choice depends only on B, L, D and the I/O dtype). A chain is 32 float32 or
+ * 64 bfloat16 channels of one batch row.
+ *   BLR_FAMILY_SERIAL     at least 256 chains: one warp walks each chain
+ *                         through the whole sequence (one kernel per call).
+ *   BLR_FAMILY_SEGMENTED  bfloat16 I/O, fewer chains, L >= 2048 and either
+ *                         at least 8 Mi elements or L >= 16384, without
+ *                         lengths: each chain is cut into time segments of
+ *                         128 steps or more; a reduction kernel computes every
+ *                         segment's affine map (the operator of Sec. 3.3),
+ *                         then one warp walks each segment from the carry the
+ *                         maps compose (two kernels per call).
+ *   BLR_FAMILY_TILED      otherwise: 64-step tiles chained by a decoupled
+ *                         look-back (a preparation kernel, then the scan).
+ *   BLR_FAMILY_NONE       an invalid or empty problem (nothing is launched).
+ */
+#define BLR_FAMILY_NONE 0
+#define BLR_FAMILY_TILED 1
+#define BLR_FAMILY_SERIAL 2
+#define BLR_FAMILY_SEGMENTED 3
+BLR_API int blr_scan_family(const blr_desc* desc, int with_lengths);
 
 /*
  * Forward BD-LRU scan (Sec. 3.2, Eq. linrnn; the scan of Sec. 3.3):

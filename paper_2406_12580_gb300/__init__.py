@@ -33,7 +33,8 @@ __all__ = [
     "BLR_F32", "BLR_BF16", "Desc", "BLRError", "blr_workspace_bytes", "blr_scan_fwd",
     "blr_scan_bwd", "blr_step", "blr_workspace_status", "blr_status_string",
     "blr_selftest_wait_timeout", "blr_scan_fwd_noalloc", "blr_scan_fwd_gated", "blr_scan_bwd_gated",
-    "blr_steps", "blr_scan_fwd_varlen", "blr_scan_bwd_varlen",
+    "blr_steps", "blr_scan_fwd_varlen", "blr_scan_bwd_varlen", "blr_scan_family",
+    "FAMILY_NONE", "FAMILY_TILED", "FAMILY_SERIAL", "FAMILY_SEGMENTED",
     "BDLRUScan", "library_loaded",
 ]
 
@@ -100,6 +101,14 @@ def _check(status: int, where: str):
 
 def blr_workspace_bytes(desc: blr_desc) -> int:
     return int(load().blr_workspace_bytes(ctypes.byref(desc)))
+
+
+# blr_scan_family results
+FAMILY_NONE, FAMILY_TILED, FAMILY_SERIAL, FAMILY_SEGMENTED = 0, 1, 2, 3
+
+
+def blr_scan_family(desc: blr_desc, with_lengths: bool = False) -> int:
+    return int(load().blr_scan_family(ctypes.byref(desc), 1 if with_lengths else 0))
 
 
 def blr_scan_fwd(desc, x, gate_logits, lam, h0, h, h_last, ws, stream=None):

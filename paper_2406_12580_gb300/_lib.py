@@ -35,6 +35,7 @@ _DESC_P = ctypes.POINTER(blr_desc)
 # name -> (restype, argtypes); the argument order of include/blr.h
 SIGNATURES = {
     "blr_workspace_bytes": (_SZ, [_DESC_P]),
+    "blr_scan_family": (ctypes.c_int, [_DESC_P, ctypes.c_int]),
     "blr_scan_fwd": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]),
     "blr_scan_bwd": (_ST, [_DESC_P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]),
     "blr_step": (_ST, [ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_float, _VP, _VP, _VP,

@@ -232,26 +232,49 @@ blr_status allow_smem(K kernel, size_t smem) {
                     "set dynamic shared memory size");
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN = false>
+// Blocks of a serial kernel: one per chain, or per (segment, chain).
+int64_t seq_blocks(const Plan& p, int mode) {
+  return mode == blr::kSeqSeg ? p.n_chain * p.nseg : p.n_chain;
+}
+
+template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE = blr::kSeqPlain>
 blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED, VARLEN>;
+  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED, MODE>;
   constexpr int NB = GATED ? 4 : 3;
-  a.stages = seq_stages(a.p.n_chain, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const int64_t blocks = seq_blocks(a.p, MODE);
+  a.stages = seq_stages(blocks, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
   const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
   BLR_TRY(allow_smem(kernel, smem));
-  kernel<<<(unsigned)a.p.n_chain, 32, smem, st>>>(a);
+  kernel<<<(unsigned)blocks, 32, smem, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch seq_fwd_kernel");
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN = false>
+template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE = blr::kSeqPlain>
 blr_status launch_seq_bwd(blr::SeqBwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED, VARLEN>;
+  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED, MODE>;
   constexpr int NB = GATED ? 5 : 4;
-  a.stages = seq_stages(a.p.n_chain, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const int64_t blocks = seq_blocks(a.p, MODE);
+  a.stages = seq_stages(blocks, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
   const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
   BLR_TRY(allow_smem(kernel, smem));
-  kernel<<<(unsigned)a.p.n_chain, 32, smem, st>>>(a);
+  kernel<<<(unsigned)blocks, 32, smem, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch seq_bwd_kernel");
+}
+
+// Rows per TMA box of the segment reductions (seg_len is a multiple).
+constexpr int kSegReduceRows = 16;
+
+template <typename T, class M, int VEC, bool BWD, bool GATED = false>
+blr_status launch_seg_reduce(blr::SegReduceArgs& a, cudaStream_t st) {
+  constexpr int R = kSegReduceRows;
+  auto kernel = blr::seg_reduce_kernel<T, M, VEC, R, BWD, GATED>;
+  constexpr int NB = (BWD && !GATED) ? 2 : 3;
+  const int64_t blocks = a.p.n_chain * a.p.nseg;
+  a.stages = seq_stages(blocks, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
+  const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
+  BLR_TRY(allow_smem(kernel, smem));
+  kernel<<<(unsigned)blocks, 32, smem, st>>>(a);
+  return cuda_check(cudaGetLastError(), "launch seg_reduce_kernel");
 }
 
 // The serial kernels' views: x-shaped tensors as (D, L, B); gate_logits-shaped
@@ -270,7 +293,7 @@ blr_status seq_maps_gl(CUtensorMap* mr, CUtensorMap* mi, const void* base, const
 // z given: the merge of the gated layer is fused, and h receives y = h SiLU(z).
 blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const float* lambda,
                         const float* h0, void* h, float* h_last, unsigned char* w, cudaStream_t st,
-                        const void* z, const int32_t* lengths) {
+                        const void* z, const int32_t* lengths, bool seg = false) {
   blr::SeqFwdArgs a;
   a.lengths = lengths;
   BLR_TRY(seq_maps_x(&a.tm_x, x, plan, plan.sr));
@@ -286,6 +309,11 @@ blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const f
   a.h_last = h_last;
   a.ws = w;
   a.stages = 2;
+  if (seg) {  // bfloat16 only (make_plan)
+    constexpr int S = blr::kSeqSeg;
+    if (z != nullptr) return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, true, S>(a, st);
+    return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, false, S>(a, st);
+  }
   if (z != nullptr) {
     if (plan.io == BLR_F32) {
       if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, true>(a, st);
@@ -294,11 +322,12 @@ blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const f
     return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, true>(a, st);
   }
   if (lengths != nullptr) {
+    constexpr int V = blr::kSeqVarlen;
     if (plan.io == BLR_F32) {
-      if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, false, true>(a, st);
-      return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16, false, true>(a, st);
+      if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, false, V>(a, st);
+      return launch_seq_fwd<float, blr::MathPrecise, 1, 16, 16, false, V>(a, st);
     }
-    return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, false, true>(a, st);
+    return launch_seq_fwd<__nv_bfloat16, blr::MathFast, 2, 16, 8, false, V>(a, st);
   }
   if (plan.io == BLR_F32) {
     if (plan.sr == 32) return launch_seq_fwd<float, blr::MathPrecise, 1, 32, 16, false>(a, st);
@@ -311,7 +340,7 @@ blr_status scan_fwd_seq(const Plan& plan, const void* x, const void* gl, const f
 blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, const void* x,
                         const void* gl, const float* lambda, const float* h0, void* dx, void* dgl,
                         float* dlambda, float* dh0, unsigned char* w, cudaStream_t st,
-                        const void* z, void* dz, const int32_t* lengths) {
+                        const void* z, void* dz, const int32_t* lengths, bool seg = false) {
   blr::SeqBwdArgs a;
   a.lengths = lengths;
   BLR_TRY(seq_maps_x(&a.tm_dh, dh, plan, plan.srb));
@@ -335,16 +364,62 @@ blr_status scan_bwd_seq(const Plan& plan, const void* dh, const float* dh_last, 
   a.dh0 = dh0;
   a.ws = w;
   a.stages = 2;
+  if (seg) {  // bfloat16 only (make_plan)
+    constexpr int S = blr::kSeqSeg;
+    if (gated) return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, true, S>(a, st);
+    return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false, S>(a, st);
+  }
   if (gated) {
     if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, true>(a, st);
     return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, true>(a, st);
   }
   if (lengths != nullptr) {
-    if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, false, true>(a, st);
-    return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false, true>(a, st);
+    constexpr int V = blr::kSeqVarlen;
+    if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, false, V>(a, st);
+    return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false, V>(a, st);
   }
   if (plan.io == BLR_F32) return launch_seq_bwd<float, blr::MathPrecise, 1, 16, 16, false>(a, st);
   return launch_seq_bwd<__nv_bfloat16, blr::MathFast, 2, 8, 8, false>(a, st);
+}
+
+// The segmented serial kernels (few chains, long sequences; bfloat16 I/O):
+// the segment reduction, then the serial kernel over (segment, chain) blocks,
+// each composing its carry from the maps.
+blr_status scan_fwd_seg(const Plan& plan, const void* x, const void* gl, const float* lambda,
+                        const float* h0, void* h, float* h_last, unsigned char* w,
+                        cudaStream_t st, const void* z) {
+  if (plan.io != BLR_BF16) return fail(BLR_ERR_UNSUPPORTED, "segmented kernels take bfloat16 I/O");
+  blr::SegReduceArgs r;
+  BLR_TRY(seq_maps_x(&r.tm_a, x, plan, kSegReduceRows));
+  BLR_TRY(seq_maps_gl(&r.tm_r, &r.tm_i, gl, plan, kSegReduceRows));
+  r.p = plan;
+  r.lambda = lambda;
+  r.ws = w;
+  r.stages = 2;
+  BLR_TRY((launch_seg_reduce<__nv_bfloat16, blr::MathFast, 2, false>(r, st)));
+  return scan_fwd_seq(plan, x, gl, lambda, h0, h, h_last, w, st, z, nullptr, true);
+}
+
+blr_status scan_bwd_seg(const Plan& plan, const void* dh, const float* dh_last, const void* x,
+                        const void* gl, const float* lambda, const float* h0, void* dx, void* dgl,
+                        float* dlambda, float* dh0, unsigned char* w, cudaStream_t st,
+                        const void* z, void* dz) {
+  if (plan.io != BLR_BF16) return fail(BLR_ERR_UNSUPPORTED, "segmented kernels take bfloat16 I/O");
+  blr::SegReduceArgs r;
+  BLR_TRY(seq_maps_x(&r.tm_a, dh, plan, kSegReduceRows));
+  BLR_TRY(seq_maps_gl(&r.tm_r, &r.tm_i, gl, plan, kSegReduceRows));
+  if (z != nullptr) BLR_TRY(seq_maps_x(&r.tm_z, z, plan, kSegReduceRows));
+  else memset(&r.tm_z, 0, sizeof(r.tm_z));
+  r.p = plan;
+  r.lambda = lambda;
+  r.ws = w;
+  r.stages = 2;
+  if (z != nullptr)
+    BLR_TRY((launch_seg_reduce<__nv_bfloat16, blr::MathFast, 2, true, true>(r, st)));
+  else
+    BLR_TRY((launch_seg_reduce<__nv_bfloat16, blr::MathFast, 2, true>(r, st)));
+  return scan_bwd_seq(plan, dh, dh_last, x, gl, lambda, h0, dx, dgl, dlambda, dh0, w, st, z, dz,
+                      nullptr, true);
 }
 
 // Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
@@ -392,7 +467,7 @@ blr_status scan_fwd_tiled(const Plan& plan, const blr_desc* desc, const void* x,
   // Clear the forward header (counters, error word), empty the
   // forward records, precompute k = -c softplus(Lambda).
   BLR_TRY(launch_prep(w + plan.off_fhdr, sizeof(blr::FwdHeader), w + plan.off_fpre,
-                      plan.off_bagg - plan.off_fpre, reinterpret_cast<float*>(w + plan.off_k),
+                      plan.off_frec_end - plan.off_fpre, reinterpret_cast<float*>(w + plan.off_k),
                       lambda, desc->D, desc->c, st));
   blr::FwdArgs a;
   a.lengths = lengths;
@@ -516,6 +591,11 @@ blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_
   if (plan.seq)  // serial kernels (the merge fused): no preparation
     return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st,
                         h != nullptr ? z : nullptr, lengths);
+  // Segmented serial kernels (the merge fused); rows with lengths on these
+  // problems run the tiled kernels.
+  if (plan.nseg > 0 && lengths == nullptr)
+    return scan_fwd_seg(plan, x, gate_logits, lambda, h0, h, h_last, w, st,
+                        h != nullptr ? z : nullptr);
   BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, h, h_last, w, st, lengths));
   if (z == nullptr || h == nullptr) return BLR_OK;
   return launch_merge_fwd(desc->io, h, z, desc->B * desc->L * desc->D, st);
@@ -564,6 +644,9 @@ blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_
   if (plan.seq)  // the forward cleared the counters and partial sums
     return scan_bwd_seq(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
                         dh0, w, st, z, dz, lengths);
+  if (plan.nseg > 0 && lengths == nullptr)
+    return scan_bwd_seg(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
+                        dh0, w, st, z, dz);
   if (z == nullptr)
     return scan_bwd_tiled(plan, desc, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
                           dlambda, dh0, w, st, lengths);
@@ -585,6 +668,15 @@ size_t blr_workspace_bytes(const blr_desc* desc) {
   bool empty = false;
   if (check_desc(desc, &plan, &empty) != BLR_OK || empty || desc->L == 0) return 0;
   return plan.bytes;
+}
+
+int blr_scan_family(const blr_desc* desc, int with_lengths) {
+  Plan plan;
+  bool empty = false;
+  if (check_desc(desc, &plan, &empty) != BLR_OK || empty || desc->L == 0) return BLR_FAMILY_NONE;
+  if (plan.seq) return BLR_FAMILY_SERIAL;
+  if (plan.nseg > 0 && !with_lengths) return BLR_FAMILY_SEGMENTED;
+  return BLR_FAMILY_TILED;
 }
 
 blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void* gate_logits,

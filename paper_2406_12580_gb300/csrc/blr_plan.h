@@ -67,6 +67,26 @@ inline int bwd_vec(int) { return 4; }
 constexpr int64_t kSeqMinChains = 256;
 constexpr int64_t kSeqTallRowsMinL = 1024;
 
+// Problems with fewer chains, bfloat16 I/O and sequences of at least kSegMinL
+// steps use the segmented serial kernels when they hold at least
+// kSegMinElems elements or L >= kSegLongL: each chain is cut into `nseg` time
+// segments of `seg_len` steps (a multiple of every box height), a reduce pass
+// computes each segment's affine map (A = prod alpha, U = its scan from a zero
+// state; for the backward W, its adjoint scan from a zero carry), and the
+// serial kernels then walk every segment from the carry that the maps of the
+// segments before it (after it, backward) compose. About kSegTargetWarps warps
+// run, 16 on each of 152 SMs; a segment is at least kSegMinLen steps.
+// Measured on GB300 against the tiled kernels: 1.45x on 8 x 32768 x 512
+// bfloat16 fwd + bwd, slower on smaller problems (fewer warps, each walking
+// at least kSegMinLen steps) and on float32 (there the reduce pass's second
+// read of the inputs costs more than the tiled kernels lose).
+constexpr int64_t kSegMinL = 2048;
+constexpr int64_t kSegMinElems = (int64_t)8 << 20;
+constexpr int64_t kSegLongL = 16384;
+constexpr int64_t kSegTargetWarps = 2432;
+constexpr int64_t kSegMinLen = 128;
+constexpr int64_t kSegAlign = 32;
+
 struct Plan {
   int64_t B, L, D;
   int io;           // 0 = float32, 1 = bfloat16
@@ -77,6 +97,8 @@ struct Plan {
   int sr, srb;      // serial: rows per TMA box, forward and backward (multiples of rb)
   int64_t n_chain;  // serial: chains = B * ceil(D / (32 * sv))
   int64_t n_carry;  // serial: kept states per chain = ceil(L / rb) - 1
+  int64_t nseg;     // segmented serial kernels: segments per chain (0: not used)
+  int64_t seg_len;  // segmented: steps per segment (the last may be shorter)
   int nwarps;       // warps per block = time sub-tiles per tile
   int64_t tsteps;   // time steps per tile = nwarps * kWarpSteps
   int64_t n_t;      // time tiles
@@ -87,8 +109,12 @@ struct Plan {
   uint32_t tag;
   // Workspace byte offsets. Records hold one entry per (time tile, channel):
   // agg = (A, U) of the tile as one 64-bit word, pre = the state after it.
-  size_t off_fhdr, off_bhdr, off_dlam, off_k;
-  size_t off_fagg, off_fpre, off_bagg, off_bpre, bytes;
+  // Segmented kernels: kept states as the serial kernels' (off_skept), the
+  // forward maps (A, U) per (segment, batch row, channel) as float pairs
+  // (off_sagg) and the backward offsets W (off_sbagg). The tiled forward
+  // records end at off_frec_end.
+  size_t off_fhdr, off_bhdr, off_dlam, off_k, off_skept, off_sagg, off_sbagg;
+  size_t off_fagg, off_fpre, off_frec_end, off_bagg, off_bpre, bytes;
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -143,6 +169,16 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   p->n_chain = B * ((D + 32 * p->sv - 1) / (32 * p->sv));
   p->n_carry = (L + p->rb - 1) / p->rb - 1;
   p->seq = p->n_chain >= kSeqMinChains ? 1 : 0;
+  p->nseg = 0;
+  p->seg_len = 0;
+  if (!p->seq && io == 1 && L >= kSegMinL && (B * L * D >= kSegMinElems || L >= kSegLongL)) {
+    int64_t n = (kSegTargetWarps + p->n_chain - 1) / p->n_chain;
+    int64_t len = (L + n - 1) / n;
+    if (len < kSegMinLen) len = kSegMinLen;
+    len = (len + kSegAlign - 1) / kSegAlign * kSegAlign;
+    p->seg_len = len;
+    p->nseg = (L + len - 1) / len;
+  }
   // The forward's states after each time tile (or every rb steps of a serial
   // chain, but the last) are kept for the backward; the tiled kernels also
   // need aggregates and backward records.
@@ -159,9 +195,20 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   p->off_k = o;
   o = align_up(o + 4 * (size_t)D, kAlign);
   p->off_fpre = o;  // forward records: pre then agg, emptied together
+  // The segmented kernels' kept states and maps lie over the tiled forward
+  // records: a forward of either family retags the workspace (the tiled one's
+  // preparation clears the tag first), and each backward checks its own tag.
+  const size_t kept_s = p->nseg ? (size_t)p->n_carry * (size_t)B * (size_t)D : 0;
+  const size_t maps_s = (size_t)p->nseg * (size_t)B * (size_t)D;
+  p->off_skept = o;
+  p->off_sagg = align_up(p->off_skept + 4 * kept_s, kAlign);
+  p->off_sbagg = align_up(p->off_sagg + 8 * maps_s, kAlign);
+  const size_t seg_end = align_up(p->off_sbagg + 4 * maps_s, kAlign);
   o = align_up(o + 4 * rec, kAlign);
   p->off_fagg = o;
   o = align_up(o + 8 * rec_t, kAlign);
+  p->off_frec_end = o;
+  if (o < seg_end) o = seg_end;
   p->off_bagg = o;  // backward records
   o = align_up(o + 8 * rec_t, kAlign);
   p->off_bpre = o;

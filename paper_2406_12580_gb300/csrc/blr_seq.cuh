@@ -115,6 +115,84 @@ struct SeqRing {
   __device__ __forceinline__ unsigned char* stage(int st) const { return base + (size_t)st * NB * BOX; }
 };
 
+// Kernel modes: the plain scan, rows with lengths, or chains cut into time
+// segments (the segmented serial kernels).
+constexpr int kSeqPlain = 0, kSeqVarlen = 1, kSeqSeg = 2;
+
+// The problem tag a segmented forward leaves in the workspace: distinct from
+// the other kernels' (its kept states and maps live elsewhere), so that a
+// segmented backward refuses a workspace that another forward filled.
+__host__ __device__ constexpr uint32_t seg_tag(uint32_t tag) { return tag ^ 0x80000000u; }
+
+// Restarts the workspace bookkeeping for a forward (one block, one warp):
+// clears the error word, the backward's exit counter and the d Lambda partial
+// sums, and tags the workspace with the problem.
+__device__ __forceinline__ void seq_reset_workspace(unsigned char* ws, const Plan& p, uint32_t tag,
+                                                    int lane) {
+  FwdHeader* fh = reinterpret_cast<FwdHeader*>(ws + p.off_fhdr);
+  BwdHeader* bh = reinterpret_cast<BwdHeader*>(ws + p.off_bhdr);
+  double* acc = reinterpret_cast<double*>(ws + p.off_dlam);
+  for (int64_t i = lane; i < (int64_t)kStripes * p.D; i += 32) acc[i] = 0.0;
+  if (lane == 0) {
+    fh->err = 0u;
+    bh->exited = 0u;
+    fh->tag = tag;
+    fh->complete = 1u;
+  }
+}
+
+// Segmented kernels. The start state of segment sg: h0 carried through the
+// maps h -> A h + U of segments 0 .. sg-1 (`agg` points at this lane's
+// channels of segment 0; segments are BD float pairs apart). Loads go out
+// eight segments at a time; missing ones are the identity map (1, 0).
+constexpr int kSegComposeBatch = 8;
+template <int VEC>
+__device__ __forceinline__ void seg_carry_in(const float2* agg, int64_t BD, int64_t sg,
+                                             float (&hc)[VEC]) {
+  constexpr int U = kSegComposeBatch;
+  for (int64_t s0 = 0; s0 < sg; s0 += U) {
+    float2 m[U][VEC];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v)
+        m[u][v] = s0 + u < sg ? __ldcg(agg + (s0 + u) * BD + v) : make_float2(1.0f, 0.0f);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) hc[v] = fmaf(m[u][v].x, hc[v], m[u][v].y);
+    }
+  }
+}
+
+// The adjoint carry at the end of segment sg: w (dh_last) carried backwards
+// through the maps w -> A w + W of segments nseg-1 .. sg+1, where A is the
+// forward map's product of alphas and W the segment's adjoint scan from a
+// zero carry (`bagg`, one float per lane channel and segment).
+template <int VEC>
+__device__ __forceinline__ void seg_adjoint_in(const float2* agg, const float* bagg, int64_t BD,
+                                               int64_t sg, int64_t nseg, float (&w)[VEC]) {
+  constexpr int U = kSegComposeBatch;
+  for (int64_t s0 = nseg - 1; s0 > sg; s0 -= U) {
+    float A[U][VEC], W[U][VEC];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int64_t s = s0 - u;
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        A[u][v] = s > sg ? __ldcg(agg + s * BD + v).x : 1.0f;
+        W[u][v] = s > sg ? __ldcg(bagg + s * BD + v) : 0.0f;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) w[v] = fmaf(A[u][v], w[v], W[u][v]);
+    }
+  }
+}
+
 // ------------------------------------------------------------------ forward
 
 // One stage, rows [0, rows) (all R when FULL). Phase 1 evaluates the
@@ -195,10 +273,14 @@ __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
   }
 }
 
-// VARLEN: the rows carry lengths (a.lengths) and each chain starts at its
-// first real step; the form without keeps the plain scan's code.
-template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN>
+// MODE kSeqVarlen: the rows carry lengths (a.lengths) and each chain starts
+// at its first real step. kSeqSeg: block (segment s, chain) walks steps
+// [s seg_len, (s + 1) seg_len) from the state that the maps (A, U) of
+// segments 0 .. s-1 (seg_reduce_kernel) carry h0 to. kSeqPlain keeps the
+// plain scan's code.
+template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE>
 __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ SeqFwdArgs a) {
+  constexpr bool VARLEN = MODE == kSeqVarlen, SEG = MODE == kSeqSeg;
   using IO = Io<T, VEC>;
   using G = typename GatePolicy<M>::type;
   constexpr int CHW = 32 * VEC;
@@ -212,33 +294,27 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
 
   const int lane = threadIdx.x;
   const int64_t n_g = (p.D + CHW - 1) / CHW;
-  const int64_t b = blockIdx.x / n_g;
-  const int64_t g = blockIdx.x - b * n_g;
+  const int64_t chain = SEG ? blockIdx.x % p.n_chain : blockIdx.x;
+  const int64_t sg = SEG ? blockIdx.x / p.n_chain : 0;
+  const int64_t b = chain / n_g;
+  const int64_t g = chain - b * n_g;
   const int64_t d0 = g * CHW + lane * VEC;
   const bool ch_ok = d0 < p.D;  // D % 8 == 0: a lane's VEC channels are all in or all out
   const int64_t BD = p.B * p.D;
   FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
-  BwdHeader* bh = reinterpret_cast<BwdHeader*>(a.ws + p.off_bhdr);
 
-  if (blockIdx.x == 0) {
-    double* acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
-    for (int64_t i = lane; i < (int64_t)kStripes * p.D; i += 32) acc[i] = 0.0;
-    if (lane == 0) {
-      fh->err = 0u;
-      bh->exited = 0u;
-      fh->tag = p.tag;
-      fh->complete = 1u;
-    }
-  }
+  if (!SEG && blockIdx.x == 0)  // the segmented reduce kernel has done this
+    seq_reset_workspace(a.ws, p, p.tag, lane);
 
   float k[VEC], kh[VEC], hc[VEC];
   const bool poly = seq_rates<VEC>(a.lambda, p.c, d0, ch_ok, k, kh);
 #pragma unroll
   for (int v = 0; v < VEC; ++v) hc[v] = (ch_ok && a.h0 != nullptr) ? a.h0[b * p.D + d0 + v] : 0.0f;
 
-  // The chain's steps: [t0, L) (all of them unless the rows carry lengths).
-  const int64_t t0 = VARLEN ? row_start(a.lengths, b, p.L) : 0;
-  const int64_t len = p.L - t0;
+  // The chain's steps: [t0, t0 + len) (all of them unless the rows carry
+  // lengths or the chain is cut into segments).
+  const int64_t t0 = SEG ? sg * p.seg_len : VARLEN ? row_start(a.lengths, b, p.L) : 0;
+  const int64_t len = SEG ? min(p.seg_len, p.L - t0) : p.L - t0;
   const int64_t nblk = (len + R - 1) / R;
   const int cd = (int)(g * CHW), cb = (int)b;
   auto issue = [&](int st, int64_t j) {
@@ -256,9 +332,13 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     for (int s = 0; s < ring.S && s < nblk; ++s) issue(s, s);
   }
   __syncwarp();
+  if constexpr (SEG) {  // while the first stages load: the segment's start state
+    if (ch_ok) seg_carry_in<VEC>(reinterpret_cast<const float2*>(a.ws + p.off_sagg) + b * p.D + d0,
+                                 BD, sg, hc);
+  }
 
-  float* carry = reinterpret_cast<float*>(a.ws + p.off_fpre) + b * p.D + d0;
-  int64_t cidx = 0;
+  float* carry = reinterpret_cast<float*>(a.ws + (SEG ? p.off_skept : p.off_fpre)) + b * p.D + d0;
+  int64_t cidx = SEG ? t0 / RB : 0;
   const int64_t n_carry = p.n_carry;
   int st = 0, prev = ring.S - 1;
   uint32_t phase = 0;
@@ -294,7 +374,7 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     }
   }
   if (lane == 0 && a.write_h) bulk_wait_all();
-  if (a.h_last != nullptr && ch_ok) {
+  if (a.h_last != nullptr && ch_ok && (!SEG || sg == p.nseg - 1)) {
 #pragma unroll
     for (int v = 0; v < VEC; ++v) a.h_last[b * p.D + d0 + v] = hc[v];
   }
@@ -417,8 +497,12 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
   }
 }
 
-template <typename T, class M, int VEC, int R, int RB, bool GATED, bool VARLEN>
+// MODE as seq_fwd_kernel's. kSeqSeg: block (segment s, chain) starts from the
+// adjoint carry that the maps (A, W) of the segments after s carry dh_last to,
+// and only segment 0 writes dh0.
+template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE>
 __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(const __grid_constant__ SeqBwdArgs a) {
+  constexpr bool VARLEN = MODE == kSeqVarlen, SEG = MODE == kSeqSeg;
   using IO = Io<T, VEC>;
   using G = typename GatePolicy<M>::type;
   constexpr int CHW = 32 * VEC;
@@ -437,14 +521,16 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   {
     int ok = 0;
     if (lane == 0) {
-      ok = __ldcg(&fh->tag) == p.tag && __ldcg(&fh->complete) == 1u;
+      ok = __ldcg(&fh->tag) == (SEG ? seg_tag(p.tag) : p.tag) && __ldcg(&fh->complete) == 1u;
       if (!ok) atomicOr(&fh->err, kErrWorkspace);
     }
     if (!__shfl_sync(kFull, ok, 0)) return;  // no forward states for this problem: write nothing
   }
   const int64_t n_g = (p.D + CHW - 1) / CHW;
-  const int64_t b = blockIdx.x / n_g;
-  const int64_t g = blockIdx.x - b * n_g;
+  const int64_t chain = SEG ? blockIdx.x % p.n_chain : blockIdx.x;
+  const int64_t sg = SEG ? blockIdx.x / p.n_chain : 0;
+  const int64_t b = chain / n_g;
+  const int64_t g = chain - b * n_g;
   const int64_t d0 = g * CHW + lane * VEC;
   const bool ch_ok = d0 < p.D;
   const int64_t BD = p.B * p.D;
@@ -459,24 +545,26 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     w[v] = (ch_ok && a.dh_last != nullptr) ? a.dh_last[b * p.D + d0 + v] : 0.0f;
     dlr[v] = 0.0f;
   }
-  const float* carry = reinterpret_cast<const float*>(a.ws + p.off_fpre) + b * p.D + d0;
-  // the state before sub-block m: h0 for m = 0, else kept state m - 1
+  const int64_t t0 = SEG ? sg * p.seg_len : VARLEN ? row_start(a.lengths, b, p.L) : 0;
+  const int64_t len = SEG ? min(p.seg_len, p.L - t0) : p.L - t0;
+  const int64_t nblk = (len + R - 1) / R;
+  const float* carry = reinterpret_cast<const float*>(a.ws + (SEG ? p.off_skept : p.off_fpre)) +
+                       b * p.D + d0;
+  const int64_t m0 = SEG ? t0 / RB : 0;  // kept states count from the chain's start
+  // the state before sub-block m of this block: h0 for the chain's first, else
+  // kept state m0 + m - 1
   auto load_start = [&](int64_t m, float (&out)[VEC]) {
 #pragma unroll
     for (int v = 0; v < VEC; ++v) {
       out[v] = 0.0f;
       if (ch_ok) {
-        if (m > 0)
-          out[v] = __ldcg(carry + (m - 1) * BD + v);
+        if (m0 + m > 0)
+          out[v] = __ldcg(carry + (m0 + m - 1) * BD + v);
         else if (a.h0 != nullptr)
           out[v] = a.h0[b * p.D + d0 + v];
       }
     }
   };
-
-  const int64_t t0 = VARLEN ? row_start(a.lengths, b, p.L) : 0;
-  const int64_t len = p.L - t0;
-  const int64_t nblk = (len + R - 1) / R;
   const int cd = (int)(g * CHW), cb = (int)b;
   auto issue = [&](int st, int64_t j) {
     unsigned char* dst = ring.stage(st);
@@ -494,6 +582,12 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     for (int s = 0; s < ring.S && s < nblk; ++s) issue(s, nblk - 1 - s);
   }
   __syncwarp();
+  if constexpr (SEG) {  // while the first stages load: the segment's end carry
+    if (ch_ok)
+      seg_adjoint_in<VEC>(reinterpret_cast<const float2*>(a.ws + p.off_sagg) + b * p.D + d0,
+                          reinterpret_cast<const float*>(a.ws + p.off_sbagg) + b * p.D + d0, BD,
+                          sg, p.nseg, w);
+  }
 
   int64_t m = (len + RB - 1) / RB - 1;  // the sub-block processed next (-1: none)
 #pragma unroll
@@ -561,7 +655,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
 
   double* acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
   if (ch_ok) {
-    if (a.dh0 != nullptr) {
+    if (a.dh0 != nullptr && (!SEG || sg == 0)) {
 #pragma unroll
       for (int v = 0; v < VEC; ++v) a.dh0[b * p.D + d0 + v] = w[v];
     }
@@ -589,6 +683,211 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
       a.dlambda[d] = (float)(-(double)p.c * sig * sum);
     }
     if (lane == 0) bh->exited = 0u;
+  }
+}
+
+// ----------------------------------------------------- segment reductions
+
+struct SegReduceArgs {
+  CUtensorMap tm_a;  // forward: x; backward: dh (gated: dy)
+  CUtensorMap tm_r;  // rho view
+  CUtensorMap tm_i;  // forward: iota view
+  CUtensorMap tm_z;  // gated backward: z
+  Plan p;
+  const float* lambda;
+  unsigned char* ws;
+  int stages;
+};
+
+// Rows [0, rows) of a forward reduce stage folded into the map (A, U): the
+// gates as seq_fwd_stage evaluates them, then h -> alpha h + u composed after
+// the map, step by step.
+template <class IO, class G, bool POLY, bool FULL, int R>
+__device__ __forceinline__ void seg_fold_fwd(const unsigned char* lb, int rows,
+                                             const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
+                                             float (&A)[IO::VEC], float (&U)[IO::VEC]) {
+  using Raw = typename IO::Raw;
+  constexpr int V = IO::VEC;
+  constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
+  constexpr uint32_t BOX = R * ROWB;
+#pragma unroll
+  for (int s = 0; s < R; ++s) {
+    if (FULL || s < rows) {
+      float xv[V], rv[V], iv[V];
+      if constexpr (G::kHalfInputs) {
+        IO::unpack_half(*reinterpret_cast<const Raw*>(lb + s * ROWB), xv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(lb + BOX + s * ROWB), rv);
+        IO::unpack_half(*reinterpret_cast<const Raw*>(lb + 2 * BOX + s * ROWB), iv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          const float e = expm1_neg<G::kDeg, POLY>(G::decay_log_half(rv[v], kh[v]));
+          const float u = G::sqrt(-e * (e + 2.0f)) * G::gated_x_half(iv[v], xv[v]);
+          U[v] = fmaf(1.0f + e, U[v], u);
+          A[v] *= 1.0f + e;
+        }
+      } else {
+        IO::unpack(*reinterpret_cast<const Raw*>(lb + s * ROWB), xv);
+        IO::unpack(*reinterpret_cast<const Raw*>(lb + BOX + s * ROWB), rv);
+        IO::unpack(*reinterpret_cast<const Raw*>(lb + 2 * BOX + s * ROWB), iv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          const float e = expm1_neg<G::kDeg, POLY>(G::decay_log(rv[v], k[v], kh[v]));
+          const float u = G::sqrt(-e * (e + 2.0f)) * (G::sigmoid(iv[v]) * xv[v]);
+          U[v] = fmaf(1.0f + e, U[v], u);
+          A[v] *= 1.0f + e;
+        }
+      }
+    }
+  }
+}
+
+// Rows [0, rows) of a backward reduce stage, last row first: w -> alpha (dh + w).
+// GATED: the first box holds dy and the third z, and dh = dy SiLU(z).
+template <class IO, class G, bool POLY, bool FULL, int R, bool GATED>
+__device__ __forceinline__ void seg_fold_bwd(const unsigned char* lb, int rows,
+                                             const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
+                                             float (&w)[IO::VEC]) {
+  using Raw = typename IO::Raw;
+  constexpr int V = IO::VEC;
+  constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
+  constexpr uint32_t BOX = R * ROWB;
+#pragma unroll
+  for (int s = R - 1; s >= 0; --s) {
+    if (FULL || s < rows) {
+      float gv[V], rv[V], l[V];
+      IO::unpack(*reinterpret_cast<const Raw*>(lb + s * ROWB), gv);
+      if constexpr (GATED) {
+        float zv[V];
+        if constexpr (G::kHalfInputs)
+          IO::unpack_half(*reinterpret_cast<const Raw*>(lb + 2 * BOX + s * ROWB), zv);
+        else
+          IO::unpack(*reinterpret_cast<const Raw*>(lb + 2 * BOX + s * ROWB), zv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) gv[v] *= G::silu(zv[v]);
+      }
+      if constexpr (G::kHalfInputs) {
+        IO::unpack_half(*reinterpret_cast<const Raw*>(lb + BOX + s * ROWB), rv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) l[v] = G::decay_log_half(rv[v], kh[v]);
+      } else {
+        IO::unpack(*reinterpret_cast<const Raw*>(lb + BOX + s * ROWB), rv);
+#pragma unroll
+        for (int v = 0; v < V; ++v) l[v] = G::decay_log(rv[v], k[v], kh[v]);
+      }
+#pragma unroll
+      for (int v = 0; v < V; ++v) w[v] = (1.0f + expm1_neg<G::kDeg, POLY>(l[v])) * (gv[v] + w[v]);
+    }
+  }
+}
+
+// Segment reductions, one warp per (segment, chain) as the segmented serial
+// kernels: the stage ring of those kernels without stores (a stage is
+// refilled as soon as every lane has read it).
+//   BWD = false: the forward map h_end = A h_start + U of the segment
+//                (x, rho, iota in), stored at off_sagg; block 0 first restarts
+//                the workspace bookkeeping for the forward.
+//   BWD = true:  the adjoint offset W = w_start for w_end = 0 (dh, rho in;
+//                GATED: dy, rho, z), stored at off_sbagg; w_start = A w_end + W
+//                with the forward's A.
+template <typename T, class M, int VEC, int R, bool BWD, bool GATED>
+__global__ void __launch_bounds__(32) seg_reduce_kernel(const __grid_constant__ SegReduceArgs a) {
+  static_assert(BWD || !GATED, "the forward map does not depend on z");
+  using IO = Io<T, VEC>;
+  using G = typename GatePolicy<M>::type;
+  constexpr int CHW = 32 * VEC;
+  constexpr int NB = (BWD && !GATED) ? 2 : 3;
+  constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
+  const Plan& p = a.p;
+  extern __shared__ unsigned char seq_smem[];
+  SeqRing<NB, BOX> ring{align128(seq_smem), nullptr, a.stages};
+  ring.bars = reinterpret_cast<uint64_t*>(ring.stage(ring.S));
+
+  const int lane = threadIdx.x;
+  const int64_t n_g = (p.D + CHW - 1) / CHW;
+  const int64_t chain = blockIdx.x % p.n_chain;
+  const int64_t sg = blockIdx.x / p.n_chain;
+  const int64_t b = chain / n_g;
+  const int64_t g = chain - b * n_g;
+  const int64_t d0 = g * CHW + lane * VEC;
+  const bool ch_ok = d0 < p.D;
+  const int64_t BD = p.B * p.D;
+  FwdHeader* fh = reinterpret_cast<FwdHeader*>(a.ws + p.off_fhdr);
+  if (!BWD && blockIdx.x == 0) seq_reset_workspace(a.ws, p, seg_tag(p.tag), lane);
+
+  float k[VEC], kh[VEC];
+  const bool poly = seq_rates<VEC>(a.lambda, p.c, d0, ch_ok, k, kh);
+  const int64_t t0 = sg * p.seg_len;
+  const int64_t len = min(p.seg_len, p.L - t0);
+  const int64_t nblk = (len + R - 1) / R;
+  const int cd = (int)(g * CHW), cb = (int)b;
+  // the forward takes the segment's stages in order, the backward from its end
+  auto blk = [&](int64_t i) { return BWD ? nblk - 1 - i : i; };
+  auto issue = [&](int st, int64_t j) {
+    unsigned char* dst = ring.stage(st);
+    const int t = (int)(t0 + j * R);
+    mbar_arrive_expect_tx(&ring.bars[st], NB * BOX);
+    tma_load_3d(dst, &a.tm_a, &ring.bars[st], cd, t, cb);
+    tma_load_3d(dst + BOX, &a.tm_r, &ring.bars[st], cd, t, cb);
+    if constexpr (!BWD) tma_load_3d(dst + 2 * BOX, &a.tm_i, &ring.bars[st], cd, t, cb);
+    if constexpr (GATED) tma_load_3d(dst + 2 * BOX, &a.tm_z, &ring.bars[st], cd, t, cb);
+  };
+  if (lane == 0) {
+    for (int s = 0; s < ring.S; ++s) mbar_init(&ring.bars[s], 1);
+    fence_mbar_init();
+    for (int s = 0; s < ring.S && s < nblk; ++s) issue(s, blk(s));
+  }
+  __syncwarp();
+
+  float A[VEC], U[VEC];  // BWD: U is w
+#pragma unroll
+  for (int v = 0; v < VEC; ++v) {
+    A[v] = 1.0f;
+    U[v] = 0.0f;
+  }
+  int st = 0;
+  uint32_t phase = 0;
+  for (int64_t i = 0; i < nblk; ++i) {
+    const int64_t j = blk(i);
+    mbar_wait(&ring.bars[st], phase, &fh->err);
+    const unsigned char* lb = ring.stage(st) + lane * VEC * sizeof(T);
+    const int64_t left = len - j * R;
+    const int rows = (int)(left < R ? left : R);
+    if constexpr (BWD) {
+      if (rows == R) {
+        if (poly)
+          seg_fold_bwd<IO, G, true, true, R, GATED>(lb, rows, k, kh, U);
+        else
+          seg_fold_bwd<IO, G, false, true, R, GATED>(lb, rows, k, kh, U);
+      } else {
+        seg_fold_bwd<IO, G, false, false, R, GATED>(lb, rows, k, kh, U);
+      }
+    } else {
+      if (rows == R) {
+        if (poly)
+          seg_fold_fwd<IO, G, true, true, R>(lb, rows, k, kh, A, U);
+        else
+          seg_fold_fwd<IO, G, false, true, R>(lb, rows, k, kh, A, U);
+      } else {
+        seg_fold_fwd<IO, G, false, false, R>(lb, rows, k, kh, A, U);
+      }
+    }
+    __syncwarp();  // every lane has read the stage: refill it
+    if (lane == 0 && i + ring.S < nblk) issue(st, blk(i + ring.S));
+    if (++st == ring.S) {
+      st = 0;
+      phase ^= 1u;
+    }
+  }
+  if (ch_ok) {
+    if constexpr (BWD) {
+      float* out = reinterpret_cast<float*>(a.ws + p.off_sbagg) + sg * BD + b * p.D + d0;
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) out[v] = U[v];
+    } else {
+      float2* out = reinterpret_cast<float2*>(a.ws + p.off_sagg) + sg * BD + b * p.D + d0;
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) out[v] = make_float2(A[v], U[v]);
+    }
   }
 }
 

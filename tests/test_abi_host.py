@@ -182,9 +182,39 @@ def test_workspace_bytes(lib):
     small, large = wb(8, 1000, 64), wb(8, 4000, 64)
     assert large > small
     assert wb(8, 4000, 64, 0, 1.0) == wb(8, 4000, 64, 0, 3.0)
-    for B, L, Dd, io in ((256, 200, 64, 0), (2048, 50, 64, 1), (64, 2048, 256, 0), (8, 32768, 512, 1)):
+    for B, L, Dd, io in ((256, 200, 64, 0), (2048, 50, 64, 1), (64, 2048, 256, 0), (8, 2047, 512, 1)):
         n = B * L * Dd
         assert wb(B, L, Dd, io) < 0.5 * n + 64 * Dd + 4096, (B, L, Dd)
+    # segmented problems keep the serial kernels' states, 12 bytes per channel
+    # per segment of 128 steps or more, and the tiled backward records
+    for B, L, Dd, io in ((8, 32768, 512, 1), (64, 2048, 64, 1), (3, 100000, 64, 1), (1, 65536, 8, 1)):
+        n = B * L * Dd
+        assert wb(B, L, Dd, io) < 0.8 * n + 24 * B * Dd + 64 * Dd + 4096, (B, L, Dd)
+
+
+def test_scan_family(lib):
+    """The kernel family follows the shape: 256 chains or more serial; fewer
+    chains, bfloat16, L >= 2048 and 8 Mi elements or L >= 16384 segmented
+    (tiled with row lengths); else tiled."""
+    fam = lambda *a, lengths=0: lib.blr_scan_family(ctypes.byref(D(*a)), lengths)  # noqa: E731
+    NONE, TILED, SERIAL, SEG = 0, 1, 2, 3
+    assert lib.blr_scan_family(None, 0) == NONE
+    assert fam(0, 10, 8) == NONE and fam(2, 0, 8) == NONE and fam(2, 10, 12) == NONE
+    assert fam(256, 200, 64) == SERIAL          # 512 float32 chains
+    assert fam(2048, 50, 64, 1) == SERIAL       # 2048 bfloat16 chains
+    assert fam(64, 2048, 256) == SERIAL
+    assert fam(255, 40000, 64, 1) == SEG        # 255 bfloat16 chains
+    assert fam(256, 40000, 64, 1) == SERIAL
+    assert fam(8, 32768, 512, 1) == SEG         # 64 bfloat16 chains
+    assert fam(8, 32768, 512, 1, lengths=1) == TILED
+    assert fam(8, 32768, 512, 0) == TILED       # float32: tiled
+    assert fam(4, 50, 64, 1) == TILED
+    assert fam(64, 2047, 64, 1) == TILED and fam(64, 2048, 64, 1) == SEG   # 8 Mi elements
+    assert fam(4, 4096, 256, 1) == TILED        # 4 Mi elements, L < 16384
+    assert fam(1, 16384, 64, 1) == SEG and fam(1, 16383, 64, 1) == TILED
+    # a bfloat16 chain is 64 channels wide: (2, 4096) float32 rows make 256
+    # chains, bfloat16 ones 128
+    assert fam(2, 4096, 4096, 0) == SERIAL and fam(2, 4096, 4096, 1) == SEG
 
 
 def test_status_strings(lib):

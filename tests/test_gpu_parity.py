@@ -345,6 +345,66 @@ def test_steps(case, io, state):
     assert torch.equal(h2, out)
 
 
+# Few chains and long bfloat16 sequences: the segmented serial kernels (time
+# segments whose maps compose the carries). A partial channel group and a
+# ragged last segment, h0 and dh_last entering through the maps, slow decays
+# and c != 1, fast decays (the e^l - 1 branch), the shortest sequence that
+# segments (at 8 Mi elements), several channel groups per row, and a chain of
+# over 300 segments.
+SEGMENTED = [
+    dict(B=1, L=16500, D=72, random_h0=True, random_dh_last=True),
+    dict(B=2, L=20000, D=64, decay=(0.99, 0.9999), c=2.0, random_dh_last=True),
+    dict(B=1, L=16384, D=256, decay=(0.05, 0.95), random_h0=True, random_dh_last=True),
+    dict(B=64, L=2048, D=64, random_h0=True),
+    dict(B=8, L=8200, D=128, random_dh_last=True),
+    dict(B=1, L=40000, D=8, decay=(0.99, 0.9999), random_h0=True, random_dh_last=True),
+]
+
+
+def _family(cfg, lengths=False):
+    from paper_2406_12580_gb300 import Desc, blr_scan_family
+    return blr_scan_family(Desc(cfg.B, cfg.L, cfg.D, 0 if cfg.io == I.F32 else 1, cfg.c), lengths)
+
+
+@pytest.mark.parametrize("case", range(len(SEGMENTED)))
+def test_segmented(case):
+    from paper_2406_12580_gb300 import FAMILY_SEGMENTED
+    inp = I.make_scan_inputs(_cfg(I.BF16, 500 + case, **SEGMENTED[case]))
+    assert _family(inp.cfg) == FAMILY_SEGMENTED
+    compare(inp, gpu_outputs(gpu_scan(inp)), oracle_outputs(inp))
+
+
+@pytest.mark.parametrize("case", [0, 2, 3])
+def test_segmented_gated(case):
+    inp = I.make_scan_inputs(_cfg(I.BF16, 520 + case, gated=True, **SEGMENTED[case]))
+    compare(inp, gpu_outputs(gpu_scan_gated(inp)), oracle_outputs(inp))
+
+
+def test_segmented_workspace_tags():
+    """A segmented backward refuses a workspace that a tiled forward of the
+    same shape filled (the _varlen forms run tiled here), and the tiled
+    backward refuses a segmented forward's."""
+    from paper_2406_12580_gb300 import (BLR_ERR_WORKSPACE, BLR_OK, FAMILY_TILED,
+                                        blr_workspace_status)
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = _cfg(I.BF16, 530, **SEGMENTED[0])
+    assert _family(cfg, lengths=True) == FAMILY_TILED
+    inp = I.make_scan_inputs(cfg)
+    buf = ScanBuffers.from_inputs(inp)
+    full = torch.full((cfg.B,), cfg.L, dtype=torch.int32, device="cuda")
+    buf.fwd_varlen(full)  # tiled kernels, all rows full length
+    buf.dx.fill_(3.0)
+    buf.bwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_ERR_WORKSPACE
+    assert torch.all(buf.dx == 3.0)
+    buf.fwd()
+    buf.bwd()
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_OK
+    compare(inp, gpu_outputs(buf), oracle_outputs(inp))
+    buf.bwd_varlen(full)  # tiled backward after a segmented forward: refused
+    assert blr_workspace_status(buf.desc, buf.ws) == BLR_ERR_WORKSPACE
+
+
 # Rows of their own lengths (blr_scan_*_varlen): sequences right-aligned in
 # their rows (left padding), padding never read or written; both kernel
 # families, empty and full rows included.
@@ -443,11 +503,14 @@ def test_fuzz(seed):
             assert normwise(got[k], w) <= tol, k
 
 
-@pytest.mark.parametrize("shape", [dict(B=300, L=130, D=40), dict(B=3, L=300, D=72)])
-def test_graph_capture_replays_eager(shape):
+@pytest.mark.parametrize("io,shape", [(I.F32, dict(B=300, L=130, D=40)),
+                                      (I.F32, dict(B=3, L=300, D=72)),
+                                      (I.BF16, dict(B=1, L=16500, D=72))])
+def test_graph_capture_replays_eager(io, shape):
     """The forward and backward captured into a CUDA graph (no host work is
-    needed between them) replay to the eager results, on both kernel families."""
-    inp = I.make_scan_inputs(_cfg(I.F32, 900, random_h0=True, random_dh_last=True, **shape))
+    needed between them) replay to the eager results, on the three kernel
+    families."""
+    inp = I.make_scan_inputs(_cfg(io, 900, random_h0=True, random_dh_last=True, **shape))
     eager = gpu_outputs(gpu_scan(inp))
     from paper_2406_12580_gb300.device import ScanBuffers
     buf = ScanBuffers.from_inputs(inp)
