@@ -68,6 +68,8 @@ def parse_args():
     ap.add_argument("--seq-len", type=int, default=0,
                     help="replace the workload's L (smaller cases for profiler captures)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--io", choices=["f32", "bf16"], default="",
+                    help="override the workload's I/O dtype (profiling other kernel families)")
     return ap.parse_args()
 
 
@@ -361,6 +363,8 @@ def run_ours(args):
     cfg = I.CONFIGS[args.config]
     if args.seq_len > 0:
         cfg = dataclasses.replace(cfg, name=f"{cfg.name} at L={args.seq_len}", L=args.seq_len)
+    if args.io and args.io != cfg.io:
+        cfg = dataclasses.replace(cfg, name=f"{cfg.name} as {args.io}", io=args.io)
     cfg = rank_workload(cfg, rank)
     inp = I.make_scan_inputs(cfg)
     buf = ScanBuffers.from_inputs(inp, device=dev)

@@ -171,6 +171,14 @@ BLR_API blr_status blr_scan_fwd(const blr_desc* desc, const void* x, const void*
  *             carries of a completed forward of the same desc, no output is
  *             written and blr_workspace_status() reports BLR_ERR_WORKSPACE. The
  *             forward's carries survive the call, so the backward may be repeated.
+ *             ws may be NULL (ws_bytes is then ignored): the call first
+ *             recomputes the forward's carries (a forward without h) in the
+ *             library's static scratch, the 128 MiB device array that
+ *             blr_scan_fwd_noalloc uses, and runs the backward from them. It
+ *             never allocates; problems whose workspace exceeds 128 MiB get
+ *             BLR_ERR_UNSUPPORTED with nothing enqueued; calls that use the
+ *             scratch must not overlap on the GPU; blr_workspace_status with
+ *             ws == NULL reads the scratch's error word.
  * h_{t-1} is recomputed from the forward's kept states, not read from h.
  */
 BLR_API blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const float* dh_last, const void* x,
@@ -191,7 +199,8 @@ BLR_API blr_status blr_scan_bwd(const blr_desc* desc, const void* dh, const floa
  *             are clamped
  * Other arguments, the workspace (sized by blr_workspace_bytes for L) and the
  * errors as blr_scan_fwd / blr_scan_bwd; the backward's ws must come from a
- * blr_scan_fwd_varlen with the same lengths. Work and traffic scale with the
+ * blr_scan_fwd_varlen with the same lengths, or be NULL (the carries are then
+ * recomputed with these lengths, as blr_scan_bwd does). Work and traffic scale with the
  * rows' lengths on problems served by the serial kernels (at least 256
  * chains); the tiled kernels still stream the padding and mask it.
  */
@@ -233,7 +242,7 @@ BLR_API blr_status blr_scan_fwd_gated(const blr_desc* desc, const void* x, const
  * z           (B, L, D)  io dtype, the forward's z
  * dz          (B, L, D)  io dtype, output
  * ws          the workspace of a blr_scan_fwd_gated (or blr_scan_fwd) of the same
- *             desc and inputs, as for blr_scan_bwd.
+ *             desc and inputs, or NULL, as for blr_scan_bwd.
  * Other arguments as blr_scan_bwd; no output may overlap an input. Problems of
  * fewer than 256 chains recompute h into dz, form dh in dx and dz in place with
  * an elementwise kernel, then run the scan's backward from dx.
@@ -281,7 +290,8 @@ BLR_API blr_status blr_steps(int64_t B, int64_t K, int64_t D, blr_dtype io, blr_
  * Synchronises `stream`, then reads the error word that the kernels of
  * earlier calls on this workspace recorded: BLR_OK, BLR_ERR_TIMEOUT or
  * BLR_ERR_WORKSPACE (BLR_ERR_CUDA if the read itself fails). The word is
- * cleared by the next blr_scan_fwd on the workspace.
+ * cleared by the next blr_scan_fwd on the workspace. ws == NULL reads the
+ * library's static scratch (that of backward calls made without a workspace).
  */
 BLR_API blr_status blr_workspace_status(const blr_desc* desc, const void* ws, size_t ws_bytes,
                                 blr_stream_t stream);
@@ -299,9 +309,9 @@ BLR_API const char* blr_last_error_string(void);
  * and serving loops that forbid allocator calls cannot provide the workspace
  * blr_scan_fwd needs. This entry point computes exactly what blr_scan_fwd
  * computes (same arguments except the workspace) on a scratch array that the
- * library holds in device memory: 64 MiB, allocated on every GPU that loads
+ * library holds in device memory: 128 MiB, allocated on every GPU that loads
  * the library and kept until the process exits. It never calls an allocator.
- *  - Problems whose workspace (blr_workspace_bytes) exceeds 64 MiB return
+ *  - Problems whose workspace (blr_workspace_bytes) exceeds 128 MiB return
  *    BLR_ERR_UNSUPPORTED with nothing enqueued; use blr_scan_fwd for them.
  *  - The first call on each device looks up the scratch array's device
  *    address (cudaGetSymbolAddress); make that first call before any stream

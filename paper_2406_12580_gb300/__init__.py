@@ -190,9 +190,11 @@ def blr_steps(B, K, D, io, state, c, h_prev, x, gate_logits, lam, h_out, h_seq=N
 
 
 def blr_workspace_status(desc, ws, stream=None) -> int:
-    """Status recorded in the workspace by earlier calls (synchronises the stream)."""
-    return int(load().blr_workspace_status(ctypes.byref(desc), _ptr(ws, "ws"), ws.numel(),
-                                           _stream(stream)))
+    """Status recorded in the workspace by earlier calls (synchronises the
+    stream); ws None reads the library's scratch (backward calls made without a
+    workspace)."""
+    return int(load().blr_workspace_status(ctypes.byref(desc), _ptr(ws, "ws"),
+                                           ws.numel() if ws is not None else 0, _stream(stream)))
 
 
 def blr_selftest_wait_timeout(desc, ws, timeout_ns: int, stream=None):

@@ -559,6 +559,12 @@ blr_status launch_merge_bwd(int io, const void* dy, const void* z, void* dh, voi
   return cuda_check(cudaGetLastError(), "launch merge_bwd_kernel");
 }
 
+// The library's static device scratch (defined with blr_scan_fwd_noalloc):
+// its size, and its address on the current device after checking that the
+// problem's workspace fits (BLR_ERR_UNSUPPORTED, nothing enqueued, if not).
+constexpr size_t kLibraryScratchBytes = (size_t)128 << 20;  // 128 MiB
+blr_status library_scratch(const Plan& plan, const char* who, void** out);
+
 // blr_scan_fwd (z == NULL) and blr_scan_fwd_gated (z given; h is then y).
 blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_logits,
                           const float* lambda, const float* h0, const void* z, void* h,
@@ -638,6 +644,16 @@ blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_
   BLR_TRY(need(gate_logits, "gate_logits", 16));
   BLR_TRY(need(dx, "dx", 16));
   BLR_TRY(need(dgate_logits, "dgate_logits", 16));
+  if (ws == nullptr) {
+    // No workspace: recompute the forward's carries (a forward without h) in
+    // the library's scratch, then run the backward from them.
+    void* scratch = nullptr;
+    BLR_TRY(library_scratch(plan, "a backward without a workspace", &scratch));
+    BLR_TRY(scan_fwd_entry(desc, x, gate_logits, lambda, h0, nullptr, nullptr, nullptr, scratch,
+                           kLibraryScratchBytes, stream, false, lengths, varlen));
+    ws = scratch;
+    ws_bytes = kLibraryScratchBytes;
+  }
   BLR_TRY(check_ws(plan, ws, ws_bytes));
 
   unsigned char* w = static_cast<unsigned char*>(ws);
@@ -813,6 +829,12 @@ blr_status blr_workspace_status(const blr_desc* desc, const void* ws, size_t ws_
   bool empty = false;
   BLR_TRY(check_desc(desc, &plan, &empty));
   if (empty || desc->L == 0) return BLR_OK;
+  if (ws == nullptr) {  // the scratch of a backward called without a workspace
+    void* scratch = nullptr;
+    BLR_TRY(library_scratch(plan, "blr_workspace_status without a workspace", &scratch));
+    ws = scratch;
+    ws_bytes = kLibraryScratchBytes;
+  }
   BLR_TRY(check_ws(plan, ws, ws_bytes));
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   uint32_t err = 0;
@@ -860,24 +882,24 @@ const char* blr_last_error_string(void) { return g_last_error; }
 }  // extern "C"
 
 // ----------------------------------------------------------------------------
-// Forward scan without a caller workspace (blr_scan_fwd_noalloc).
+// Scans without a caller workspace (blr_scan_fwd_noalloc, and the backward
+// entry points given ws == NULL).
 //
 // Some callers cannot allocate device memory at the point where they run the
 // scan: code inside CUDA stream capture that may not add allocations, plugins
 // whose host framework owns every device allocation, or real-time serving
-// loops that forbid allocator calls. For them the forward scan can run on a
-// scratch array that lives in the library itself: a file-scope device array
-// of kNoAllocScratchBytes, present on every GPU that loads this library until
+// loops that forbid allocator calls. For them the scan can run on a scratch
+// array that lives in the library itself: a file-scope device array of
+// kLibraryScratchBytes, present on every GPU that loads this library until
 // the process exits. The host never dereferences the array's name (in host
 // code it is only a stand-in for the device symbol); the device address comes
 // from cudaGetSymbolAddress, once per device.
 
 namespace {
 
-constexpr size_t kNoAllocScratchBytes = (size_t)64 << 20;  // 64 MiB
 constexpr int kMaxDevices = 64;
 
-__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+__device__ __align__(256) unsigned char g_noalloc_scratch[kLibraryScratchBytes];
 
 std::mutex g_scratch_mutex;
 void* g_scratch_ptr[kMaxDevices] = {};
@@ -900,6 +922,15 @@ blr_status noalloc_scratch(void** out) {
   return BLR_OK;
 }
 
+blr_status library_scratch(const Plan& plan, const char* who, void** out) {
+  if (plan.bytes > kLibraryScratchBytes)
+    return fail(BLR_ERR_UNSUPPORTED,
+                "%s: this problem needs %zu bytes of scratch, above the %zu-byte static scratch; "
+                "pass a workspace of blr_workspace_bytes",
+                who, plan.bytes, kLibraryScratchBytes);
+  return noalloc_scratch(out);
+}
+
 }  // namespace
 
 extern "C" blr_status blr_scan_fwd_noalloc(const blr_desc* desc, const void* x,
@@ -911,14 +942,8 @@ extern "C" blr_status blr_scan_fwd_noalloc(const blr_desc* desc, const void* x,
   BLR_TRY(check_desc(desc, &plan, &empty));
   if (empty || desc->L == 0)  // nothing that needs scratch: the ordinary path does it
     return blr_scan_fwd(desc, x, gate_logits, lambda, h0, h, h_last, nullptr, 0, stream);
-  const size_t need_bytes = plan.bytes;
-  if (need_bytes > kNoAllocScratchBytes)
-    return fail(BLR_ERR_UNSUPPORTED,
-                "blr_scan_fwd_noalloc: this problem needs %zu bytes of scratch, above the %zu-byte "
-                "static scratch; use blr_scan_fwd with a caller workspace",
-                need_bytes, kNoAllocScratchBytes);
   void* scratch = nullptr;
-  BLR_TRY(noalloc_scratch(&scratch));
-  return blr_scan_fwd(desc, x, gate_logits, lambda, h0, h, h_last, scratch, kNoAllocScratchBytes,
+  BLR_TRY(library_scratch(plan, "blr_scan_fwd_noalloc", &scratch));
+  return blr_scan_fwd(desc, x, gate_logits, lambda, h0, h, h_last, scratch, kLibraryScratchBytes,
                       stream);
 }

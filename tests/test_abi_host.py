@@ -105,8 +105,15 @@ def bwd(lib, desc, **kw):
 def test_bwd_validation(lib):
     assert bwd(lib, D(2, 4, 12)) == _lib.BLR_ERR_UNSUPPORTED
     assert bwd(lib, D(2, 4, 8, c=-1.0)) == _lib.BLR_ERR_INVALID_ARG
-    for name in ("dh", "x", "gl", "lam", "dx", "dgl", "dlam", "ws"):
+    for name in ("dh", "x", "gl", "lam", "dx", "dgl", "dlam"):
         assert bwd(lib, D(2, 4, 8), **{name: None}) == _lib.BLR_ERR_INVALID_ARG, name
+    # without a workspace the backward recomputes the carries in the library's
+    # 128 MiB scratch; a problem that does not fit is refused before anything
+    # is enqueued
+    big = D(64, 100000, 512)
+    assert lib.blr_workspace_bytes(ctypes.byref(big)) > (128 << 20)
+    assert bwd(lib, big, ws=None, ws_bytes=0) == _lib.BLR_ERR_UNSUPPORTED
+    assert b"static scratch" in lib.blr_last_error_string()
     for name in ("dh", "x", "gl", "dx", "dgl", "lam"):
         assert bwd(lib, D(2, 4, 8), **{name: FAKE + 8}) == _lib.BLR_ERR_INVALID_ARG, name
     for name in ("dh_last", "h0", "dh0", "dlam"):

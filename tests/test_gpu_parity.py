@@ -405,6 +405,64 @@ def test_segmented_workspace_tags():
     assert blr_workspace_status(buf.desc, buf.ws) == BLR_ERR_WORKSPACE
 
 
+@pytest.mark.parametrize("io,shape", [(I.F32, dict(B=300, L=130, D=40)),
+                                      (I.F32, dict(B=3, L=300, D=72)),
+                                      (I.BF16, dict(B=1, L=16500, D=72))])
+def test_backward_without_workspace(io, shape):
+    """ws = NULL: the backward recomputes the forward's carries in the library's
+    scratch and gives the results of a backward from the forward's workspace,
+    plain, gated and with row lengths, on the three kernel families."""
+    from paper_2406_12580_gb300 import (BLR_OK, blr_scan_bwd, blr_scan_bwd_gated,
+                                        blr_scan_bwd_varlen, blr_workspace_status)
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = _cfg(io, 950, random_h0=True, random_dh_last=True, **shape)
+    inp = I.make_scan_inputs(cfg)
+    buf = ScanBuffers.from_inputs(inp)
+    lengths = torch.from_numpy(np.random.default_rng(3).integers(0, cfg.L + 1, size=cfg.B)
+                               .astype(np.int32)).cuda()
+    outs = lambda: [t.clone() for t in (buf.dx, buf.dgl, buf.dlam, buf.dh0)]  # noqa: E731
+    z = torch.randn_like(buf.x)
+    dz = torch.zeros_like(buf.x)
+    for mode in ("plain", "gated", "varlen"):
+        for t in (buf.dx, buf.dgl, dz):
+            t.zero_()
+        if mode == "plain":
+            buf.fwd()
+            buf.bwd()
+        elif mode == "gated":
+            buf.fwd()  # a plain forward's workspace serves the gated backward
+            blr_scan_bwd_gated(buf.desc, buf.dh, buf.dh_last, buf.x, buf.gl, buf.lam, buf.h0, z,
+                               buf.dx, buf.dgl, dz, buf.dlam, buf.dh0, buf.ws)
+        else:
+            buf.fwd_varlen(lengths)
+            buf.bwd_varlen(lengths)
+        torch.cuda.synchronize()
+        want = outs() + ([dz.clone()] if mode == "gated" else [])
+        for t in (buf.dx, buf.dgl, buf.dlam, buf.dh0, dz):
+            t.fill_(7.0)
+        buf.ws.zero_()  # nothing of the forward is left for the backward
+        if mode == "plain":
+            blr_scan_bwd(buf.desc, buf.dh, buf.dh_last, buf.x, buf.gl, buf.lam, buf.h0, buf.dx,
+                         buf.dgl, buf.dlam, buf.dh0, None)
+        elif mode == "gated":
+            blr_scan_bwd_gated(buf.desc, buf.dh, buf.dh_last, buf.x, buf.gl, buf.lam, buf.h0, z,
+                               buf.dx, buf.dgl, dz, buf.dlam, buf.dh0, None)
+        else:
+            for t in (buf.dx, buf.dgl):
+                t.copy_(want[0] if t is buf.dx else want[1])  # the padding is never written
+            blr_scan_bwd_varlen(buf.desc, lengths, buf.dh, buf.dh_last, buf.x, buf.gl, buf.lam,
+                                buf.h0, buf.dx, buf.dgl, buf.dlam, buf.dh0, None)
+        torch.cuda.synchronize()
+        assert blr_workspace_status(buf.desc, None) == BLR_OK
+        got = outs() + ([dz.clone()] if mode == "gated" else [])
+        for g, w in zip(got, want):
+            # the same kernels: float32 results agree up to the order of float
+            # atomics and of the tiled look-back's combines, which can move a
+            # bfloat16 output by one unit in its last place
+            tol = 2.0 ** -7 if g.dtype == torch.bfloat16 else 1e-6
+            assert normwise(g.float().cpu().numpy(), w.float().cpu().numpy()) <= tol, mode
+
+
 # Rows of their own lengths (blr_scan_*_varlen): sequences right-aligned in
 # their rows (left padding), padding never read or written; both kernel
 # families, empty and full rows included.
