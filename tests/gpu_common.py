@@ -114,14 +114,29 @@ def oracle_outputs(inp: I.ScanInputs, dsel=None, threads=0):
     return out
 
 
+def elementwise(got, want) -> float:
+    """Diagnostic beside the normwise error: max |gpu - oracle| / (|oracle| +
+    1e-3 max|oracle|), relative per element but defined at exact zeros."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    if want.size == 0:
+        return 0.0
+    floor = 1e-3 * np.max(np.abs(want))
+    if floor == 0.0:
+        return float(np.max(np.abs(got - want)))
+    return float(np.max(np.abs(got - want) / (np.abs(want) + floor)))
+
+
 def compare(inp: I.ScanInputs, got: dict, want: dict, tol=None):
+    """Asserts the normwise error of every output; returns it with the
+    elementwise diagnostic ({name: (normwise, elementwise)})."""
     tol = TOL[inp.cfg.io] if tol is None else tol
     errs = {}
     for k, w in want.items():
         errs[k] = normwise(got[k], w)
     bad = {k: v for k, v in errs.items() if not v <= tol}
     assert not bad, f"{inp.cfg.name}: normwise errors above {tol}: {bad} (all: {errs})"
-    return errs
+    return {k: (v, elementwise(got[k], want[k])) for k, v in errs.items()}
 
 
 def gpu_step(sinp: I.StepInputs):

@@ -304,6 +304,73 @@ def test_gated_long_sequence_sampled():
     print(f"gated config 4: {errs}")
 
 
+@pytest.mark.parametrize("io", [I.F32, I.BF16])
+def test_gate_math_against_cuda(io):
+    """The device gate arithmetic against CUDA's own functions. The step kernel
+    evaluates the gates with the same primitives as the scans (sigmoid from
+    ex2.approx and rcp.approx in float32, from tanh.approx in the bfloat16
+    path; e^l - 1 by its Taylor series where |l| < 0.25, ex2 - 1 beyond;
+    sqrt.approx): with h_prev = 1 and x = 0 a step returns alpha, with h_prev = 0
+    and x = 1 it returns sqrt(1 - alpha^2) i. Both are compared with the same
+    quantities from torch's CUDA float32 operators (expm1f, sigmoid, sqrtf) and
+    with float64, over logits in [-30, 30] plus saturating ones, decays
+    exp(-softplus(Lambda)) in [0.05, 0.9999] and c in {0.5, 1, 3, 8}.
+    Bounds: float32, |d alpha| <= 1e-6 and |d(beta i)| <= (4e-6 + 1e-7 (|rho| +
+    |iota|)) |beta i| + 1e-12 (a few units of 2^-23 through each step, and the
+    rounding of the sigmoids' exponents); bfloat16, from tanh.approx's
+    relative error 2^-11, r and i are off by at most 2^-12, so
+    |d alpha| <= |k| 2^-12 + 5e-5 (k = -c softplus(Lambda); 5e-5 covers the
+    degree-4 series) and |d(beta i)| <= sqrt(2 |d alpha|) + 2^-12."""
+    from paper_2406_12580_gb300 import blr_step, _dtype_code
+    B, D = 2048, 64
+    g = torch.Generator().manual_seed(11)
+    rho = torch.linspace(-30.0, 30.0, B, dtype=torch.float64)
+    rho[:8] = torch.tensor([-1e4, -200.0, -80.0, -40.0, 40.0, 80.0, 200.0, 1e4], dtype=torch.float64)
+    iota = rho[torch.randperm(B, generator=g)]
+    u = torch.linspace(0.05, 0.9999, D, dtype=torch.float64)
+    lam = torch.log((1.0 - u) / u).float()
+    tdt = torch.float32 if io == I.F32 else torch.bfloat16
+    gl = torch.cat([rho[:, None].expand(B, D), iota[:, None].expand(B, D)], dim=1).to(tdt)
+    rr, ii = gl[:, :D].double().cpu(), gl[:, D:].double().cpu()  # the rounded logits both sides see
+    dev = "cuda"
+    gl_d, lam_d = gl.to(dev).contiguous(), lam.to(dev)
+    ones = torch.ones(B, D, device=dev)
+    zeros = torch.zeros(B, D, device=dev)
+    x0, x1 = torch.zeros(B, D, dtype=tdt, device=dev), torch.ones(B, D, dtype=tdt, device=dev)
+    for c in (0.5, 1.0, 3.0, 8.0):
+        alpha, bi = torch.empty(B, D, device=dev), torch.empty(B, D, device=dev)
+        blr_step(B, D, _dtype_code(gl_d), c, ones, x0, gl_d, lam_d, alpha)
+        blr_step(B, D, _dtype_code(gl_d), c, zeros, x1, gl_d, lam_d, bi)
+        torch.cuda.synchronize()
+        alpha, bi = alpha.double().cpu(), bi.double().cpu()
+        assert torch.isfinite(alpha).all() and torch.isfinite(bi).all(), c
+        k64 = -c * torch.nn.functional.softplus(lam.double())[None, :]
+        l64 = k64 * torch.sigmoid(rr)
+        a64 = torch.exp(l64)
+        bi64 = torch.sqrt(-torch.expm1(2.0 * l64)) * torch.sigmoid(ii)
+        # CUDA's float32 functions on the same logits
+        r32 = torch.sigmoid(rr.float().to(dev))
+        l32 = (-c * torch.nn.functional.softplus(lam_d))[None, :] * r32
+        e32 = torch.expm1(l32)
+        a32 = (1.0 + e32).double().cpu()
+        bi32 = (torch.sqrt(-e32 * (2.0 + e32)) * torch.sigmoid(ii.float().to(dev))).double().cpu()
+        da, dbi = (alpha - a64).abs(), (bi - bi64).abs()
+        if io == I.F32:
+            bound_a = torch.full_like(da, 1e-6)
+            # the exponent z log2(e) of the sigmoids is rounded too: 2^-24 |z|
+            # relative in each sigmoid, which grows with the logit
+            bound_bi = (4e-6 + 1e-7 * (rr.abs() + ii.abs())) * bi64.abs() + 1e-12
+        else:
+            bound_a = k64.abs().expand(B, D) * 2.0 ** -12 + 5e-5
+            bound_bi = torch.sqrt(2.0 * bound_a) + 2.0 ** -12
+        worst_a = float((da / bound_a).max())
+        worst_bi = float((dbi / bound_bi).max())
+        print(f"{io} c={c}: |d alpha| max {float(da.max()):.2e} (CUDA f32 {float((a32 - a64).abs().max()):.2e}), "
+              f"|d(beta i)| max {float(dbi.max()):.2e} (CUDA f32 {float((bi32 - bi64).abs().max()):.2e}); "
+              f"worst error / bound {worst_a:.3f}, {worst_bi:.3f}")
+        assert worst_a <= 1.0 and worst_bi <= 1.0, (io, c, worst_a, worst_bi)
+
+
 # K recurrent steps per row (blr_steps): io and state dtypes crossed, with and
 # without the per-step states, the last state written over the first.
 STEPS = [dict(B=1, L=1, D=8), dict(B=3, L=5, D=72), dict(B=1000, L=16, D=64, c=2.0),
