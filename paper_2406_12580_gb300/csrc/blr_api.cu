@@ -237,13 +237,23 @@ int64_t seq_blocks(const Plan& p, int mode) {
   return mode == blr::kSeqSeg ? p.n_chain * p.nseg : p.n_chain;
 }
 
+// float32 rings deep enough run the LATE form (refill after the next stage's
+// arithmetic); bfloat16 always the early one.
+template <typename T>
+bool late_refill(int stages) {
+  return sizeof(T) == 4 && stages >= blr::kSeqLateRefillStages;
+}
+
 template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE = blr::kSeqPlain>
 blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED, MODE>;
   constexpr int NB = GATED ? 4 : 3;
   const int64_t blocks = seq_blocks(a.p, MODE);
   a.stages = seq_stages(blocks, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
   const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
+  auto kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED, MODE, false>;
+  if constexpr (sizeof(T) == 4) {
+    if (late_refill<T>(a.stages)) kernel = blr::seq_fwd_kernel<T, M, VEC, R, RB, GATED, MODE, true>;
+  }
   BLR_TRY(allow_smem(kernel, smem));
   kernel<<<(unsigned)blocks, 32, smem, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch seq_fwd_kernel");
@@ -251,11 +261,14 @@ blr_status launch_seq_fwd(blr::SeqFwdArgs& a, cudaStream_t st) {
 
 template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE = blr::kSeqPlain>
 blr_status launch_seq_bwd(blr::SeqBwdArgs& a, cudaStream_t st) {
-  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED, MODE>;
   constexpr int NB = GATED ? 5 : 4;
   const int64_t blocks = seq_blocks(a.p, MODE);
   a.stages = seq_stages(blocks, NB * (size_t)blr::seq_box_bytes<T, VEC, R>());
   const size_t smem = blr::seq_smem_bytes<T, VEC, R>(a.stages, NB);
+  auto kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED, MODE, false>;
+  if constexpr (sizeof(T) == 4) {
+    if (late_refill<T>(a.stages)) kernel = blr::seq_bwd_kernel<T, M, VEC, R, RB, GATED, MODE, true>;
+  }
   BLR_TRY(allow_smem(kernel, smem));
   kernel<<<(unsigned)blocks, 32, smem, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch seq_bwd_kernel");

@@ -33,6 +33,12 @@
 namespace blr {
 
 constexpr int kSeqMaxStages = 8;   // ring stages per warp
+// Rings of at least this many stages may refill a consumed stage after the
+// next stage's arithmetic rather than before it (the kernels' LATE form;
+// measured on GB300: float32 rings of 4-8 stages up to 5 % faster that way,
+// bfloat16 rings of 2-3 stages 3-7 % slower, so bfloat16 keeps the early
+// form).
+constexpr int kSeqLateRefillStages = 4;
 
 // Tensor maps: (channels, time, batch) views with boxes of 32 * VEC channels x
 // R steps x 1 row. gate_logits is seen as two views of D channels each
@@ -278,7 +284,8 @@ __device__ __forceinline__ void seq_fwd_stage(unsigned char* sb, int rows,
 // [s seg_len, (s + 1) seg_len) from the state that the maps (A, U) of
 // segments 0 .. s-1 (seg_reduce_kernel) carry h0 to. kSeqPlain keeps the
 // plain scan's code.
-template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE>
+// LATE: refill a consumed stage after the next stage's arithmetic (deep rings).
+template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE, bool LATE>
 __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ SeqFwdArgs a) {
   constexpr bool VARLEN = MODE == kSeqVarlen, SEG = MODE == kSeqSeg;
   using IO = Io<T, VEC>;
@@ -344,8 +351,9 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
   uint32_t phase = 0;
   for (int64_t j = 0; j < nblk; ++j) {
     mbar_wait(&ring.bars[st], phase, &fh->err);
-    // the previous stage's store has read it by now (or shortly will): refill it
-    if (lane == 0 && j > 0 && j - 1 + ring.S < nblk) {
+    // Shallow rings refill the previous stage at the top of the iteration, deep
+    // ones after this stage's arithmetic (as the backward).
+    if (!LATE && lane == 0 && j > 0 && j - 1 + ring.S < nblk) {
       if (a.write_h) bulk_wait_read<0>();
       issue(prev, j - 1 + ring.S);
     }
@@ -363,9 +371,15 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     }
     fence_proxy_async_smem();  // the stage's h rows, visible to the TMA store
     __syncwarp();
-    if (lane == 0 && a.write_h) {
-      tma_store_3d(&a.tm_h, sb, cd, (int)(t0 + j * R), cb);
-      bulk_commit();
+    if (lane == 0) {
+      if (LATE && j > 0 && j - 1 + ring.S < nblk) {
+        if (a.write_h) bulk_wait_read<0>();
+        issue(prev, j - 1 + ring.S);
+      }
+      if (a.write_h) {
+        tma_store_3d(&a.tm_h, sb, cd, (int)(t0 + j * R), cb);
+        bulk_commit();
+      }
     }
     prev = st;
     if (++st == ring.S) {
@@ -500,7 +514,7 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
 // MODE as seq_fwd_kernel's. kSeqSeg: block (segment s, chain) starts from the
 // adjoint carry that the maps (A, W) of the segments after s carry dh_last to,
 // and only segment 0 writes dh0.
-template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE>
+template <typename T, class M, int VEC, int R, int RB, bool GATED, int MODE, bool LATE>
 __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(const __grid_constant__ SeqBwdArgs a) {
   constexpr bool VARLEN = MODE == kSeqVarlen, SEG = MODE == kSeqSeg;
   using IO = Io<T, VEC>;
@@ -601,8 +615,10 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   for (int64_t i = 0; i < nblk; ++i) {
     const int64_t j = nblk - 1 - i;
     mbar_wait(&ring.bars[st], phase, &fh->err);
-    // the previous stage's stores have read it by now (or shortly will): refill it
-    if (lane == 0 && i > 0 && i - 1 + ring.S < nblk) {
+    // Shallow rings refill the previous stage as soon as its stores have read
+    // it, at the top of the iteration; deep ones after this stage's arithmetic,
+    // when those stores are long done and the wait costs nothing.
+    if (!LATE && lane == 0 && i > 0 && i - 1 + ring.S < nblk) {
       bulk_wait_read<0>();
       issue(prev, nblk - 1 - (i - 1 + ring.S));
     }
@@ -638,6 +654,10 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
     fence_proxy_async_smem();  // the stage's outputs, visible to the TMA stores
     __syncwarp();
     if (lane == 0) {
+      if (LATE && i > 0 && i - 1 + ring.S < nblk) {
+        bulk_wait_read<0>();
+        issue(prev, nblk - 1 - (i - 1 + ring.S));
+      }
       const int t = (int)(t0 + j * R);
       tma_store_3d(&a.tm_dx, sb, cd, t, cb);
       tma_store_3d(&a.tm_dr, sb + 2 * BOX, cd, t, cb);
