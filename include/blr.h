@@ -224,9 +224,10 @@ BLR_API blr_status blr_scan_bwd_varlen(const blr_desc* desc, const int32_t* leng
  * y           (B, L, D)  io dtype, output; may be NULL (then only h_last and
  *                        the carries, as blr_scan_fwd with h == NULL)
  * Other arguments, the workspace and the errors as blr_scan_fwd; z must be
- * 16-byte aligned and no output may overlap an input. Problems of fewer than
- * 256 chains (batch rows x groups of 32 float32 / 64 bfloat16 channels) run
- * the scan and then an elementwise merge kernel over y in place.
+ * 16-byte aligned and no output may overlap an input. The merge is fused into
+ * the serial and segmented kernels; problems on the tiled kernels
+ * (blr_scan_family) run the scan and then an elementwise merge kernel over y
+ * in place.
  */
 BLR_API blr_status blr_scan_fwd_gated(const blr_desc* desc, const void* x, const void* gate_logits,
                                       const float* lambda, const float* h0, const void* z, void* y,
@@ -243,9 +244,10 @@ BLR_API blr_status blr_scan_fwd_gated(const blr_desc* desc, const void* x, const
  * dz          (B, L, D)  io dtype, output
  * ws          the workspace of a blr_scan_fwd_gated (or blr_scan_fwd) of the same
  *             desc and inputs, or NULL, as for blr_scan_bwd.
- * Other arguments as blr_scan_bwd; no output may overlap an input. Problems of
- * fewer than 256 chains recompute h into dz, form dh in dx and dz in place with
- * an elementwise kernel, then run the scan's backward from dx.
+ * Other arguments as blr_scan_bwd; no output may overlap an input. Problems on
+ * the tiled kernels (blr_scan_family) recompute h into dz, form dh in dx and dz
+ * in place with an elementwise kernel, then run the scan's backward from dx;
+ * the serial and segmented kernels fuse the merge.
  */
 BLR_API blr_status blr_scan_bwd_gated(const blr_desc* desc, const void* dy, const float* dh_last,
                                       const void* x, const void* gate_logits, const float* lambda,

@@ -44,7 +44,7 @@ SMALL = [
     dict(B=600, L=100, D=72, random_h0=True, random_dh_last=True),
     dict(B=520, L=129, D=32, decay=(0.99, 0.9999)),
     # fast decays (exp(-softplus(Lambda)) down to 0.05, so |log alpha| > 0.25:
-    # the general e^l - 1 branch) and c != 1, on both kernel families
+    # the general e^l - 1 branch) and c != 1, on the serial and tiled families
     dict(B=3, L=150, D=40, decay=(0.05, 0.95), c=3.0, random_h0=True, random_dh_last=True),
     dict(B=400, L=90, D=40, decay=(0.05, 0.95), c=0.5, random_h0=True, random_dh_last=True),
     # a long sequence with many chains (float32: the forward's 32-row boxes),
