@@ -769,22 +769,26 @@ blr_status blr_step(int64_t B, int64_t D, blr_dtype io, float c, const float* h_
   BLR_TRY(need(gate_logits_t, "gate_logits_t", 16));
   BLR_TRY(need(lambda, "lambda", 16));
   BLR_TRY(need(h_t, "h_t", 16));
-  constexpr int kRows = 4;
+  // f32: two rows of 4 channels a thread per step of its walk; bf16: one row of 8
+  const int rows = (io == BLR_F32) ? 2 : 1;
   const int vec = (io == BLR_F32) ? 4 : 8;
   const int64_t nvec = D / vec;
   const int bx = (int)(nvec < 64 ? nvec : 64);
   const int by = 256 / bx;
   const int64_t n_vgroups = (nvec + bx - 1) / bx;
-  const int64_t rows_per_block = (int64_t)by * kRows;
-  const int64_t n_rgroups = (B + rows_per_block - 1) / rows_per_block;
-  if (n_vgroups * n_rgroups >= ((int64_t)1 << 31)) return fail(BLR_ERR_UNSUPPORTED, "grid too large");
+  // a persistent grid: as many row groups as fill the GPU, at most one per block row of work
+  const int64_t need_rg = (B + (int64_t)by * rows - 1) / ((int64_t)by * rows);
+  int64_t n_rg = ((int64_t)sm_count() * blr::kStepBlocksPerSm + n_vgroups - 1) / n_vgroups;
+  if (n_rg > need_rg) n_rg = need_rg;
+  if (n_rg < 1) n_rg = 1;
+  if (n_vgroups * n_rg >= ((int64_t)1 << 31)) return fail(BLR_ERR_UNSUPPORTED, "grid too large");
   blr::StepArgs a{B, D, c, n_vgroups, h_prev, x_t, gate_logits_t, lambda, h_t};
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 grid((unsigned)(n_vgroups * n_rgroups)), block((unsigned)bx, (unsigned)by);
+  const dim3 grid((unsigned)(n_vgroups * n_rg)), block((unsigned)bx, (unsigned)by);
   if (io == BLR_F32)
-    blr::step_kernel<float, 4, blr::MathPrecise, kRows><<<grid, block, 0, st>>>(a);
+    blr::step_kernel<float, 4, blr::MathPrecise, 2><<<grid, block, 0, st>>>(a);
   else
-    blr::step_kernel<__nv_bfloat16, 8, blr::MathFast, kRows><<<grid, block, 0, st>>>(a);
+    blr::step_kernel<__nv_bfloat16, 8, blr::MathFast, 1><<<grid, block, 0, st>>>(a);
   return cuda_check(cudaGetLastError(), "launch step_kernel");
 }
 

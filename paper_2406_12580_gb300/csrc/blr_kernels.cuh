@@ -991,16 +991,21 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 3)
 
 // ------------------------------------------------------------ recurrent step
 //
-// h_t = alpha h_prev + beta x for B rows of D channels. A block covers
-// blockDim.x channel vectors of blockDim.y * ROWS rows; k = -c softplus(Lambda)
-// is computed once per channel per block.
+// h_t = alpha h_prev + beta x for B rows of D channels. A persistent grid: a
+// block covers blockDim.x channel vectors and computes k = -c softplus(Lambda)
+// for them once; each thread then walks rows ROWS at a time, with a stride of
+// the grid's row threads, loading the next rows' inputs before the current
+// rows' arithmetic so that every thread keeps loads in flight.
+
+constexpr int kStepBlocksPerSm = 3;
 
 template <typename T, int VEC, class M, int ROWS>
-__global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
+__global__ void __launch_bounds__(256, kStepBlocksPerSm) step_kernel(const StepArgs a) {
   using IO = Io<T, VEC>;
   __shared__ float s_k[64 * 8];
   const int64_t vg = blockIdx.x % a.n_vgroups;
   const int64_t rg = blockIdx.x / a.n_vgroups;
+  const int64_t n_rg = gridDim.x / a.n_vgroups;  // the grid launches whole channel groups
   const int64_t dblock = vg * blockDim.x * VEC;
   const int tid = threadIdx.y * blockDim.x + threadIdx.x;
   for (int j = tid; j < (int)blockDim.x * VEC; j += blockDim.x * blockDim.y)
@@ -1008,37 +1013,57 @@ __global__ void __launch_bounds__(256) step_kernel(const StepArgs a) {
   __syncthreads();
   const int64_t d0 = dblock + threadIdx.x * VEC;
   if (d0 >= a.D) return;
-  const int64_t r0 = (rg * blockDim.y + threadIdx.y) * ROWS;
+  float k[VEC];
+#pragma unroll
+  for (int v = 0; v < VEC; ++v) k[v] = s_k[threadIdx.x * VEC + v];
   const T* x = static_cast<const T*>(a.x);
   const T* gl = static_cast<const T*>(a.gl);
+  const int64_t rstride = n_rg * blockDim.y * ROWS;  // rows the grid takes per step of the walk
   float hp[ROWS][VEC], xv[ROWS][VEC], rv[ROWS][VEC], iv[ROWS][VEC];
+  auto load = [&](int64_t r0) {
 #pragma unroll
-  for (int r = 0; r < ROWS; ++r) {
-    const int64_t bb = r0 + r;
-    if (bb < a.B) {
-      load_f32<VEC>(a.h_prev + bb * a.D + d0, hp[r]);
-      IO::unpack(IO::load_raw(x + bb * a.D + d0), xv[r]);
-      IO::unpack(IO::load_raw(gl + bb * 2 * a.D + d0), rv[r]);
-      IO::unpack(IO::load_raw(gl + bb * 2 * a.D + a.D + d0), iv[r]);
+    for (int r = 0; r < ROWS; ++r) {
+      const int64_t bb = r0 + r;
+      if (bb < a.B) {
+        load_f32<VEC>(a.h_prev + bb * a.D + d0, hp[r]);
+        IO::unpack(IO::load_raw(x + bb * a.D + d0), xv[r]);
+        IO::unpack(IO::load_raw(gl + bb * 2 * a.D + d0), rv[r]);
+        IO::unpack(IO::load_raw(gl + bb * 2 * a.D + a.D + d0), iv[r]);
+      }
     }
-  }
+  };
+  int64_t r0 = (rg * blockDim.y + threadIdx.y) * ROWS;
+  if (r0 < a.B) load(r0);
+  for (; r0 < a.B; r0 += rstride) {
+    float ch[ROWS][VEC], cx[ROWS][VEC], cr[ROWS][VEC], ci[ROWS][VEC];
 #pragma unroll
-  for (int r = 0; r < ROWS; ++r) {
-    const int64_t bb = r0 + r;
-    if (bb < a.B) {
-      float out[VEC];
+    for (int r = 0; r < ROWS; ++r) {
 #pragma unroll
       for (int v = 0; v < VEC; ++v) {
-        const float k = s_k[threadIdx.x * VEC + v];
-        const float rr = M::sigmoid(rv[r][v]);
-        const float i = M::sigmoid(iv[r][v]);
-        const float e = M::expm1_any(k * rr);
-        out[v] = fmaf(1.0f + e, hp[r][v], M::sqrt(-e * (2.0f + e)) * i * xv[r][v]);
+        ch[r][v] = hp[r][v];
+        cx[r][v] = xv[r][v];
+        cr[r][v] = rv[r][v];
+        ci[r][v] = iv[r][v];
       }
+    }
+    if (r0 + rstride < a.B) load(r0 + rstride);  // in flight during this rows' arithmetic
 #pragma unroll
-      for (int j = 0; j < VEC; j += 4)
-        __stcs(reinterpret_cast<float4*>(a.h_t + bb * a.D + d0 + j),
-               make_float4(out[j], out[j + 1], out[j + 2], out[j + 3]));
+    for (int r = 0; r < ROWS; ++r) {
+      const int64_t bb = r0 + r;
+      if (bb < a.B) {
+        float out[VEC];
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) {
+          const float rr = M::sigmoid(cr[r][v]);
+          const float i = M::sigmoid(ci[r][v]);
+          const float e = M::expm1_any(k[v] * rr);
+          out[v] = fmaf(1.0f + e, ch[r][v], M::sqrt(-e * (2.0f + e)) * i * cx[r][v]);
+        }
+#pragma unroll
+        for (int j = 0; j < VEC; j += 4)
+          __stcs(reinterpret_cast<float4*>(a.h_t + bb * a.D + d0 + j),
+                 make_float4(out[j], out[j + 1], out[j + 2], out[j + 3]));
+      }
     }
   }
 }
