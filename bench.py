@@ -474,30 +474,32 @@ def run_ours(args):
     return 0
 
 
-def e2e_pipelined(inp, reps, world, dev):
+def e2e_pipelined(inp, reps, world, dev, nsets=3):
     """Same metric through the C ABI with host buffers, steps streamed: every
-    step copies its inputs from pinned host memory and reads every output back;
-    step k+1's host-to-device copies run on their own stream beside step k's
-    scan and device-to-host copies (two device buffer sets, alternating)."""
+    step copies its inputs from pinned host memory and reads every output back.
+    Three streams — host-to-device copies, the scan, device-to-host copies —
+    and `nsets` device buffer sets in rotation, so that step k's outputs go
+    back while step k+1 computes and step k+2's inputs arrive."""
     import torch
     from paper_2406_12580_gb300.device import ScanBuffers, to_device
     cfg = inp.cfg
     pin = lambda name: to_device(inp.io_array(name), cfg.io, "cpu", pin=False).pin_memory()  # noqa: E731
     hx, hgl, hdh = pin("x"), pin("gl"), pin("dh") if not cfg.fwd_only else None
-    bufs = [ScanBuffers.from_inputs(inp, device=dev) for _ in range(2)]
+    bufs = [ScanBuffers.from_inputs(inp, device=dev) for _ in range(nsets)]
     outs = [[b.h, b.h_last] + ([] if cfg.fwd_only else [b.dx, b.dgl, b.dlam]) for b in bufs]
     host_outs = [[torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs[0]]
-                 for _ in range(2)]
+                 for _ in range(nsets)]
     h2d = sum(t.numel() * t.element_size() for t in (hx, hgl, hdh) if t is not None)
     d2h = sum(t.numel() * t.element_size() for t in host_outs[0])
-    s_in, s_run = torch.cuda.Stream(), torch.cuda.Stream()
-    done = [None, None]
+    s_in, s_run, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    freed = [None] * nsets  # set j's outputs copied back: its buffers are free again
 
     def step(k):
-        b, j = bufs[k % 2], k % 2
+        j = k % nsets
+        b = bufs[j]
         with torch.cuda.stream(s_in):
-            if done[j] is not None:
-                s_in.wait_event(done[j])  # the buffers' previous step is finished with them
+            if freed[j] is not None:
+                s_in.wait_event(freed[j])
             b.x.copy_(hx, non_blocking=True)
             b.gl.copy_(hgl, non_blocking=True)
             if hdh is not None:
@@ -509,26 +511,32 @@ def e2e_pipelined(inp, reps, world, dev):
             b.fwd()
             if not cfg.fwd_only:
                 b.bwd()
+            computed = torch.cuda.Event()
+            computed.record(s_run)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(computed)
             for d, o in zip(host_outs[j], outs[j]):
                 d.copy_(o, non_blocking=True)
-            done[j] = torch.cuda.Event()
-            done[j].record(s_run)
+            freed[j] = torch.cuda.Event()
+            freed[j].record(s_out)
 
-    for k in range(3):
+    for k in range(nsets + 1):
         step(k)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(s_in)
     s_run.wait_event(e0)
+    s_out.wait_event(e0)
     for k in range(reps):
         step(k)
-    e1.record(s_run)
+    e1.record(s_out)  # after the last step's copies back, which follow all of its work
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / reps
     return {"value": world * cfg.elements / (ms * 1e-3), "unit": UNIT, "ms_per_step": ms,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "pipelining": "step k+1's host-to-device copies overlap step k's scan and "
-                          "device-to-host copies (two streams, two buffer sets; more copy streams measured no faster)"}
+            "pipelining": (f"three streams (copies in, scan, copies out) and {nsets} device buffer "
+                           "sets: step k's copies back overlap step k+1's scan and step k+2's "
+                           "copies in")}
 
 
 def e2e(buf, inp, reps, world):
