@@ -97,10 +97,11 @@ typedef struct {
  *           element;
  *   tiled: per-tile records (24 bytes per channel per 64-step tile, under 0.4
  *           bytes per element);
- *   segmented: the serial kernels' kept states and 12 bytes per channel per
- *           segment (of 128 steps or more), laid over the tiled forward
+ *   segmented: the serial kernels' kept states, 8 bytes per channel per
+ *           segment (of 128 steps or more) and the chained forward's records
+ *           (12 bytes per channel per 64 steps), laid over the tiled forward
  *           records, plus the tiled backward records (for the _varlen forms),
- *           under 0.8 bytes per element;
+ *           under 0.95 bytes per element;
  * plus the float64 partial sums of dlambda and a small header (about 72 bytes
  * per channel). It depends only on B, L, D and the I/O dtype.
  */

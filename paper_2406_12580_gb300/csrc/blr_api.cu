@@ -12,6 +12,7 @@
 #include <cudaTypedefs.h>
 
 #include "blr.h"
+#include "blr_chain.cuh"
 #include "blr_merge.cuh"
 #include "blr_seq.cuh"
 
@@ -60,6 +61,8 @@ blr_status check_desc(const blr_desc* d, Plan* plan, bool* empty_bd) {
   blr::make_plan(d->B, d->L, d->D, (int)d->io, d->c, plan);
   if (plan->n_tiles_f >= ((int64_t)1 << 30) || plan->n_tiles_b >= ((int64_t)1 << 30))
     return fail(BLR_ERR_UNSUPPORTED, "too many tiles (%lld)", (long long)plan->n_tiles_b);
+  if (plan->nseg > 0 && plan->n_tc * plan->n_chain >= ((int64_t)1 << 31))
+    return fail(BLR_ERR_UNSUPPORTED, "too many chained tiles");
   if (plan->seq && plan->n_chain >= ((int64_t)1 << 31))
     return fail(BLR_ERR_UNSUPPORTED, "too many chains (%lld)", (long long)plan->n_chain);
   return BLR_OK;
@@ -435,6 +438,36 @@ blr_status scan_bwd_seg(const Plan& plan, const void* dh, const float* dh_last, 
                       nullptr, true);
 }
 
+// The chained single-pass forward (few chains, long sequences): its records
+// are emptied, then one cooperative grid, one block per SM, scans every tile.
+template <typename T, class M, int VEC, int RB>
+blr_status launch_chain_fwd(const Plan& plan, const blr::ChainFwdArgs& a, cudaStream_t st) {
+  constexpr int threads = blr::kChainThreads;
+  auto k = blr::chain_fwd_kernel<T, M, VEC, RB>;
+  const size_t smem = blr::ChainSmem<T, VEC>::bytes;
+  unsigned grid = 1;
+  BLR_TRY(persistent_grid(k, threads, smem, plan.n_tc * plan.n_chain, &grid));
+  return launch_cooperative(k, grid, threads, smem, st, a, "launch chain_fwd_kernel");
+}
+
+blr_status scan_fwd_chain(const Plan& plan, const void* x, const void* gl, const float* lambda,
+                          const float* h0, void* h, float* h_last, unsigned char* w,
+                          cudaStream_t st) {
+  BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_cinc, 0xff, plan.off_cend - plan.off_cinc, st),
+                     "empty the chained forward's records"));
+  blr::ChainFwdArgs a;
+  BLR_TRY(seq_maps_x(&a.tm_x, x, plan, blr::kChainTile));
+  BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, blr::kChainTile));
+  a.p = plan;
+  a.lambda = lambda;
+  a.h0 = h0;
+  a.h = h;
+  a.h_last = h_last;
+  a.ws = w;
+  if (plan.io == BLR_F32) return launch_chain_fwd<float, blr::MathPrecise, 1, 16>(plan, a, st);
+  return launch_chain_fwd<__nv_bfloat16, blr::MathFast, 2, 8>(plan, a, st);
+}
+
 // Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
 // empty record pattern and writes k = -c softplus(Lambda).
 blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fill,
@@ -610,11 +643,15 @@ blr_status scan_fwd_entry(const blr_desc* desc, const void* x, const void* gate_
   if (plan.seq)  // serial kernels (the merge fused): no preparation
     return scan_fwd_seq(plan, x, gate_logits, lambda, h0, h, h_last, w, st,
                         h != nullptr ? z : nullptr, lengths);
-  // Segmented serial kernels (the merge fused); rows with lengths on these
-  // problems run the tiled kernels.
-  if (plan.nseg > 0 && lengths == nullptr)
-    return scan_fwd_seg(plan, x, gate_logits, lambda, h0, h, h_last, w, st,
-                        h != nullptr ? z : nullptr);
+  // Few long chains: the chained single-pass forward, or with the gated
+  // layer's merge the segmented serial kernels (the merge fused); rows with
+  // lengths on these problems run the tiled kernels. Either forward leaves the
+  // kept states the segmented backward starts from.
+  if (plan.nseg > 0 && lengths == nullptr) {
+    if (z == nullptr || h == nullptr)
+      return scan_fwd_chain(plan, x, gate_logits, lambda, h0, h, h_last, w, st);
+    return scan_fwd_seg(plan, x, gate_logits, lambda, h0, h, h_last, w, st, z);
+  }
   BLR_TRY(scan_fwd_tiled(plan, desc, x, gate_logits, lambda, h0, h, h_last, w, st, lengths));
   if (z == nullptr || h == nullptr) return BLR_OK;
   return launch_merge_fwd(desc->io, h, z, desc->B * desc->L * desc->D, st);

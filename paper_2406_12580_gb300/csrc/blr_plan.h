@@ -80,6 +80,15 @@ constexpr int64_t kSeqTallRowsMinL = 1024;
 // bfloat16 fwd + bwd, slower on smaller problems (fewer warps, each walking
 // at least kSegMinLen steps) and on float32 (there the reduce pass's second
 // read of the inputs costs more than the tiled kernels lose).
+// The forward of those problems runs a chained single-pass kernel instead of
+// the reduction and the serial pass (the backward keeps the segmented
+// kernels): tiles of kChainTile steps x one chain, kChainWarps compute warps a
+// tile (a warp slice of kChainSlice steps), chained along time by a decoupled
+// look-back over per-(tile, channel) records.
+constexpr int kChainWarps = 16;
+constexpr int kChainSlice = 4;
+constexpr int kChainTile = kChainWarps * kChainSlice;
+
 constexpr int64_t kSegMinL = 2048;
 constexpr int64_t kSegMinElems = (int64_t)8 << 20;
 constexpr int64_t kSegLongL = 16384;
@@ -99,6 +108,7 @@ struct Plan {
   int64_t n_carry;  // serial: kept states per chain = ceil(L / rb) - 1
   int64_t nseg;     // segmented serial kernels: segments per chain (0: not used)
   int64_t seg_len;  // segmented: steps per segment (the last may be shorter)
+  int64_t n_tc;     // chained forward (when nseg > 0): time blocks of kChainTile steps
   int nwarps;       // warps per block = time sub-tiles per tile
   int64_t tsteps;   // time steps per tile = nwarps * kWarpSteps
   int64_t n_t;      // time tiles
@@ -109,11 +119,14 @@ struct Plan {
   uint32_t tag;
   // Workspace byte offsets. Records hold one entry per (time tile, channel):
   // agg = (A, U) of the tile as one 64-bit word, pre = the state after it.
-  // Segmented kernels: kept states as the serial kernels' (off_skept), the
-  // forward maps (A, U) per (segment, batch row, channel) as float pairs
-  // (off_sagg) and the backward offsets W (off_sbagg). The tiled forward
-  // records end at off_frec_end.
-  size_t off_fhdr, off_bhdr, off_dlam, off_k, off_skept, off_sagg, off_sbagg;
+  // Segmented kernels: kept states as the serial kernels' (off_skept) and one
+  // map per (segment, batch row, channel) as a float pair (off_sagg: the
+  // forward's (A, U) within a gated forward call, the backward's (A, W)).
+  // Chained forward: its records, the state after each tile (off_cinc, 32-bit)
+  // then the tile's map (off_cagg, 64-bit), filled with ones together before
+  // each call.
+  // The tiled forward records end at off_frec_end.
+  size_t off_fhdr, off_bhdr, off_dlam, off_k, off_skept, off_sagg, off_cinc, off_cagg, off_cend;
   size_t off_fagg, off_fpre, off_frec_end, off_bagg, off_bpre, bytes;
 };
 
@@ -171,6 +184,7 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   p->seq = p->n_chain >= kSeqMinChains ? 1 : 0;
   p->nseg = 0;
   p->seg_len = 0;
+  p->n_tc = 0;
   if (!p->seq && io == 1 && L >= kSegMinL && (B * L * D >= kSegMinElems || L >= kSegLongL)) {
     int64_t n = (kSegTargetWarps + p->n_chain - 1) / p->n_chain;
     int64_t len = (L + n - 1) / n;
@@ -178,6 +192,7 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
     len = (len + kSegAlign - 1) / kSegAlign * kSegAlign;
     p->seg_len = len;
     p->nseg = (L + len - 1) / len;
+    p->n_tc = (L + kChainTile - 1) / kChainTile;
   }
   // The forward's states after each time tile (or every rb steps of a serial
   // chain, but the last) are kept for the backward; the tiled kernels also
@@ -200,10 +215,13 @@ inline void make_plan(int64_t B, int64_t L, int64_t D, int io, float c, Plan* p)
   // preparation clears the tag first), and each backward checks its own tag.
   const size_t kept_s = p->nseg ? (size_t)p->n_carry * (size_t)B * (size_t)D : 0;
   const size_t maps_s = (size_t)p->nseg * (size_t)B * (size_t)D;
+  const size_t crec = (size_t)p->n_tc * (size_t)B * (size_t)D;
   p->off_skept = o;
   p->off_sagg = align_up(p->off_skept + 4 * kept_s, kAlign);
-  p->off_sbagg = align_up(p->off_sagg + 8 * maps_s, kAlign);
-  const size_t seg_end = align_up(p->off_sbagg + 4 * maps_s, kAlign);
+  p->off_cinc = align_up(p->off_sagg + 8 * maps_s, kAlign);
+  p->off_cagg = align_up(p->off_cinc + 4 * crec, kAlign);
+  p->off_cend = align_up(p->off_cagg + 8 * crec, kAlign);
+  const size_t seg_end = p->off_cend;
   o = align_up(o + 4 * rec, kAlign);
   p->off_fagg = o;
   o = align_up(o + 8 * rec_t, kAlign);

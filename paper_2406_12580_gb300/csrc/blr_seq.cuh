@@ -174,27 +174,25 @@ __device__ __forceinline__ void seg_carry_in(const float2* agg, int64_t BD, int6
 
 // The adjoint carry at the end of segment sg: w (dh_last) carried backwards
 // through the maps w -> A w + W of segments nseg-1 .. sg+1, where A is the
-// forward map's product of alphas and W the segment's adjoint scan from a
-// zero carry (`bagg`, one float per lane channel and segment).
+// segment's product of alphas and W its adjoint scan from a zero carry (one
+// float pair (A, W) per lane channel and segment, written by the backward's
+// segment reduction).
 template <int VEC>
-__device__ __forceinline__ void seg_adjoint_in(const float2* agg, const float* bagg, int64_t BD,
-                                               int64_t sg, int64_t nseg, float (&w)[VEC]) {
+__device__ __forceinline__ void seg_adjoint_in(const float2* maps, int64_t BD, int64_t sg,
+                                               int64_t nseg, float (&w)[VEC]) {
   constexpr int U = kSegComposeBatch;
   for (int64_t s0 = nseg - 1; s0 > sg; s0 -= U) {
-    float A[U][VEC], W[U][VEC];
+    float2 m[U][VEC];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int64_t s = s0 - u;
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        A[u][v] = s > sg ? __ldcg(agg + s * BD + v).x : 1.0f;
-        W[u][v] = s > sg ? __ldcg(bagg + s * BD + v) : 0.0f;
-      }
+      for (int v = 0; v < VEC; ++v) m[u][v] = s > sg ? __ldcg(maps + s * BD + v) : make_float2(1.0f, 0.0f);
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) w[v] = fmaf(A[u][v], w[v], W[u][v]);
+      for (int v = 0; v < VEC; ++v) w[v] = fmaf(m[u][v].x, w[v], m[u][v].y);
     }
   }
 }
@@ -598,8 +596,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   __syncwarp();
   if constexpr (SEG) {  // while the first stages load: the segment's end carry
     if (ch_ok)
-      seg_adjoint_in<VEC>(reinterpret_cast<const float2*>(a.ws + p.off_sagg) + b * p.D + d0,
-                          reinterpret_cast<const float*>(a.ws + p.off_sbagg) + b * p.D + d0, BD,
+      seg_adjoint_in<VEC>(reinterpret_cast<const float2*>(a.ws + p.off_sagg) + b * p.D + d0, BD,
                           sg, p.nseg, w);
   }
 
@@ -761,12 +758,13 @@ __device__ __forceinline__ void seg_fold_fwd(const unsigned char* lb, int rows,
   }
 }
 
-// Rows [0, rows) of a backward reduce stage, last row first: w -> alpha (dh + w).
-// GATED: the first box holds dy and the third z, and dh = dy SiLU(z).
+// Rows [0, rows) of a backward reduce stage, last row first: w -> alpha (dh + w),
+// and the product A of the alphas. GATED: the first box holds dy and the third
+// z, and dh = dy SiLU(z).
 template <class IO, class G, bool POLY, bool FULL, int R, bool GATED>
 __device__ __forceinline__ void seg_fold_bwd(const unsigned char* lb, int rows,
                                              const float (&k)[IO::VEC], const float (&kh)[IO::VEC],
-                                             float (&w)[IO::VEC]) {
+                                             float (&A)[IO::VEC], float (&w)[IO::VEC]) {
   using Raw = typename IO::Raw;
   constexpr int V = IO::VEC;
   constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
@@ -795,7 +793,11 @@ __device__ __forceinline__ void seg_fold_bwd(const unsigned char* lb, int rows,
         for (int v = 0; v < V; ++v) l[v] = G::decay_log(rv[v], k[v], kh[v]);
       }
 #pragma unroll
-      for (int v = 0; v < V; ++v) w[v] = (1.0f + expm1_neg<G::kDeg, POLY>(l[v])) * (gv[v] + w[v]);
+      for (int v = 0; v < V; ++v) {
+        const float alpha = 1.0f + expm1_neg<G::kDeg, POLY>(l[v]);
+        w[v] = alpha * (gv[v] + w[v]);
+        A[v] *= alpha;
+      }
     }
   }
 }
@@ -806,9 +808,10 @@ __device__ __forceinline__ void seg_fold_bwd(const unsigned char* lb, int rows,
 //   BWD = false: the forward map h_end = A h_start + U of the segment
 //                (x, rho, iota in), stored at off_sagg; block 0 first restarts
 //                the workspace bookkeeping for the forward.
-//   BWD = true:  the adjoint offset W = w_start for w_end = 0 (dh, rho in;
-//                GATED: dy, rho, z), stored at off_sbagg; w_start = A w_end + W
-//                with the forward's A.
+//   BWD = true:  the adjoint map w_start = A w_end + W of the segment: A the
+//                product of its alphas, W = w_start for w_end = 0 (dh, rho in;
+//                GATED: dy, rho, z), stored at off_sagg over the forward's maps,
+//                which only the forward call itself uses.
 template <typename T, class M, int VEC, int R, bool BWD, bool GATED>
 __global__ void __launch_bounds__(32) seg_reduce_kernel(const __grid_constant__ SegReduceArgs a) {
   static_assert(BWD || !GATED, "the forward map does not depend on z");
@@ -858,7 +861,7 @@ __global__ void __launch_bounds__(32) seg_reduce_kernel(const __grid_constant__ 
   }
   __syncwarp();
 
-  float A[VEC], U[VEC];  // BWD: U is w
+  float A[VEC], U[VEC];  // BWD: U is W
 #pragma unroll
   for (int v = 0; v < VEC; ++v) {
     A[v] = 1.0f;
@@ -875,11 +878,11 @@ __global__ void __launch_bounds__(32) seg_reduce_kernel(const __grid_constant__ 
     if constexpr (BWD) {
       if (rows == R) {
         if (poly)
-          seg_fold_bwd<IO, G, true, true, R, GATED>(lb, rows, k, kh, U);
+          seg_fold_bwd<IO, G, true, true, R, GATED>(lb, rows, k, kh, A, U);
         else
-          seg_fold_bwd<IO, G, false, true, R, GATED>(lb, rows, k, kh, U);
+          seg_fold_bwd<IO, G, false, true, R, GATED>(lb, rows, k, kh, A, U);
       } else {
-        seg_fold_bwd<IO, G, false, false, R, GATED>(lb, rows, k, kh, U);
+        seg_fold_bwd<IO, G, false, false, R, GATED>(lb, rows, k, kh, A, U);
       }
     } else {
       if (rows == R) {
@@ -899,15 +902,9 @@ __global__ void __launch_bounds__(32) seg_reduce_kernel(const __grid_constant__ 
     }
   }
   if (ch_ok) {
-    if constexpr (BWD) {
-      float* out = reinterpret_cast<float*>(a.ws + p.off_sbagg) + sg * BD + b * p.D + d0;
+    float2* out = reinterpret_cast<float2*>(a.ws + p.off_sagg) + sg * BD + b * p.D + d0;
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) out[v] = U[v];
-    } else {
-      float2* out = reinterpret_cast<float2*>(a.ws + p.off_sagg) + sg * BD + b * p.D + d0;
-#pragma unroll
-      for (int v = 0; v < VEC; ++v) out[v] = make_float2(A[v], U[v]);
-    }
+    for (int v = 0; v < VEC; ++v) out[v] = make_float2(A[v], U[v]);
   }
 }
 

@@ -657,6 +657,10 @@ def test_graph_capture_replays_eager(io, shape):
     torch.cuda.synchronize()
     got = gpu_outputs(buf)
     # the same kernels, so the same values up to the order of float atomics
-    # (dLambda) and of look-back combines (the tiled kernels)
+    # (dLambda) and of look-back combines: a look-back folds whichever
+    # predecessors have published when it reads, so float32 carries may differ
+    # in their last bits between calls, and a bfloat16 output by one rounding
+    # step (2^-8 of its magnitude) where such a carry sits at a rounding boundary
+    tol = 1e-6 if io == I.F32 else 2.0 ** -8
     for k in eager:
-        assert normwise(got[k], eager[k]) <= 1e-6, k
+        assert normwise(got[k], eager[k]) <= tol, k
