@@ -3,16 +3,24 @@
 
 One step = one forward scan plus one backward scan (the whole training hot
 path: gates, decay and input normalisation, forward scan, reverse scan,
-dLambda) over one batch of synthetic input, the B=256, L=200, D=64 float32
-workload (ML-1M's maximum length and the paper's embedding width). Inputs are
-resident in HBM when the timed region starts; L2 is flushed (a 2x L2 write)
-before every timed step; each step is timed on the device with CUDA events.
+dLambda) over one batch of synthetic input. The headline workload is the
+long-sequence one, B=8, L=32768, D=512, bfloat16 I/O with float32 state
+(XLong-like histories scaled up): its inputs (2.9 GB a step) are larger than
+L2, so K steps run back to back between two CUDA events, each C-ABI call also
+bracketed by its own events for the per-kernel roofline. Inputs are resident
+in HBM when the timed region starts.
+
+The other workloads are reported beside it, each with its own roofline
+(`configs`): they fit L2, so L2 is flushed (a 2x L2 write) before every timed
+call, the backward's included.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--config 0-4] [--extras]
 
-Prints one JSON line on rank 0. Under torchrun each rank runs its own replica
-of the workload (the scan shards over batch rows and channels with no
-exchange), so the value is the sum over ranks ("weak" scaling).
+Prints one JSON line on rank 0 (--extras: a second line with further
+workloads on stderr). Under torchrun each rank runs its own replica of the
+workload (the scan shards over batch rows and channels with no exchange), so
+the value is the sum over ranks ("weak" scaling).
 
 --impl reference times the float64 CPU oracle, as it stands, on the host
 cores (there is no other implementation of this method to compare against).
@@ -60,11 +68,13 @@ def log(*a):
 def parse_args():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=1, help="workload (0-4); 1 is the headline")
+    ap.add_argument("--config", type=int, default=4, help="workload (0-4); 4 is the headline")
     ap.add_argument("--quick", action="store_true", help="skip the other workloads and e2e")
+    ap.add_argument("--extras", action="store_true",
+                    help="also time the gated, varlen, K-step and layer workloads (stderr)")
     ap.add_argument("--seq-len", type=int, default=0,
                     help="replace the workload's L (smaller cases for profiler captures)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -121,18 +131,34 @@ def kernel_sources_sha() -> str:
 
 
 def scan_kernels(cfg):
-    """(forward kernels, backward kernels, launches per call, what a call's
-    CUDA events bracket) of the family the library runs on this shape
-    (blr_scan_family)."""
+    """(forward kernels, backward kernels, our kernels per forward call, per
+    backward call) of the family the library runs on this shape
+    (blr_scan_family). The chained forward also clears its records with one
+    cudaMemsetAsync, which is not counted as a kernel of ours."""
     from paper_2406_12580_gb300 import (FAMILY_SEGMENTED, FAMILY_SERIAL, Desc,
                                         blr_scan_family)
     fam = blr_scan_family(Desc(cfg.B, cfg.L, cfg.D, 0 if cfg.io == "f32" else 1, cfg.c))
     if fam == FAMILY_SERIAL:
-        return "seq_fwd_kernel", "seq_bwd_kernel", 1, "the kernel alone"
+        return "seq_fwd_kernel", "seq_bwd_kernel", 1, 1
     if fam == FAMILY_SEGMENTED:
-        return ("seg_reduce_kernel+seq_fwd_kernel", "seg_reduce_kernel+seq_bwd_kernel", 2,
-                "the segment reduction and the serial kernel")
-    return "scan_fwd_kernel", "scan_bwd_kernel", 2, "the kernel and its preparation kernel"
+        return "chain_fwd_kernel", "seg_reduce_kernel+seq_bwd_kernel", 1, 2
+    return "prep_kernel+scan_fwd_kernel", "prep_kernel+scan_bwd_kernel", 2, 2
+
+
+def config_dict(cfg, world: int, l2: str) -> dict:
+    """The `config` object of the JSON line (the same for both arms)."""
+    return {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io,
+            "state": "f32", "parallelism": f"replicas{world}" if world > 1 else "single",
+            "l2": l2, "inputs": "seeded synthetic (paper_2406_12580_gb300.inputs), resident in HBM"}
+
+
+def l2_policy(cfg, l2_bytes: int):
+    """(flush between timed calls?, description): workloads whose per-step
+    traffic exceeds twice the L2 run back to back, the others flush L2."""
+    step_bytes = cfg.elements * (FWD_VALUES + BWD_VALUES) * io_bytes(cfg.io)
+    if step_bytes > 2 * l2_bytes:
+        return False, f"inputs larger than L2 ({step_bytes / 1e9:.2f} GB a step): no flush"
+    return True, f"flushed before every timed call ({2 * l2_bytes >> 20} MiB write)"
 
 
 def ncu_traffic(kernel: str, workload: str):
@@ -235,6 +261,19 @@ def cpu_oracle_rate(inp, target_s: float = 10.0, max_reps: int = 1000, threads: 
 
 # --------------------------------------------------------------- reference
 
+def nominal_l2_bytes() -> int:
+    """L2 size of the device if torch can see one, else GB300's 129 MiB."""
+    try:
+        import torch
+        if torch.cuda.is_available():
+            v = int(getattr(torch.cuda.get_device_properties(0), "L2_cache_size", 0) or 0)
+            if v > 0:
+                return v
+    except Exception:
+        pass
+    return 129 << 20
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -245,20 +284,24 @@ def run_reference(args):
     cfg = I.CONFIGS[args.config]
     threads = os.cpu_count() or 1
     # One reference step = fwd + bwd of the oracle over a bounded sample of the
-    # workload (whole batch rows), sized to about one second.
-    probe = I.make_scan_inputs(I.scaled(cfg, B=max(1, min(cfg.B, 8))))
+    # workload (whole batch rows), sized so that warm-up and timed steps take
+    # about two minutes in all.
+    per_step_s = min(1.0, 120.0 / max(1, args.steps + args.warmup))
+    probe_rows = 1 if cfg.L * cfg.D > (1 << 20) else max(1, min(cfg.B, 8))
+    probe = I.make_scan_inputs(I.scaled(cfg, B=probe_rows))
     t = time.perf_counter()
-    orc.fwd(probe.x, probe.gl, probe.lam, probe.h0, threads=threads)
+    orc.fwd(probe.x, probe.gl, probe.lam, probe.h0, c=cfg.c, threads=threads)
     if probe.dh is not None:
-        orc.bwd(probe.dh, probe.x, probe.gl, probe.lam, probe.h0, probe.dh_last, threads=threads)
+        orc.bwd(probe.dh, probe.x, probe.gl, probe.lam, probe.h0, probe.dh_last, c=cfg.c,
+                threads=threads)
     per_row = (time.perf_counter() - t) / probe.cfg.B
-    Bs = int(max(1, min(cfg.B, 1.0 / max(per_row, 1e-9))))
-    inp = I.make_scan_inputs(I.scaled(cfg, B=Bs))
+    Bs = int(max(1, min(cfg.B, per_step_s / max(per_row, 1e-9))))
+    inp = probe if Bs == probe_rows else I.make_scan_inputs(I.scaled(cfg, B=Bs))
 
     def step():
-        orc.fwd(inp.x, inp.gl, inp.lam, inp.h0, threads=threads)
+        orc.fwd(inp.x, inp.gl, inp.lam, inp.h0, c=cfg.c, threads=threads)
         if inp.dh is not None:
-            orc.bwd(inp.dh, inp.x, inp.gl, inp.lam, inp.h0, inp.dh_last, threads=threads)
+            orc.bwd(inp.dh, inp.x, inp.gl, inp.lam, inp.h0, inp.dh_last, c=cfg.c, threads=threads)
 
     for _ in range(args.warmup):
         step()
@@ -273,7 +316,7 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io},
+        "config": config_dict(cfg, args.gpus, l2_policy(cfg, nominal_l2_bytes())[1]),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads if orc.has_openmp else 1,
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -284,27 +327,33 @@ def run_reference(args):
 
 # -------------------------------------------------------------------- ours
 
-def time_scan(buf, reps, flush, with_bwd=True):
-    """Per-rep device time (ms) of the forward and the backward, L2 flushed
-    before each rep."""
+def time_calls(buf, reps, flush=None, with_bwd=True):
+    """Times `reps` steps (forward, then backward) with CUDA events on the
+    launching stream: per call, and, when nothing runs between the steps
+    (flush is None), the whole region. With `flush`, L2 is flushed before
+    every call. Returns (fwd ms list, bwd ms list, region ms or None)."""
     import torch
-    fwd_ms, bwd_ms = [], []
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-           torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
-    for k in range(reps):
-        flush()
-        e0, e1, e2 = ev[k]
+    E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    ev = [(E(), E(), E(), E()) for _ in range(reps)]
+    r0, r1 = E(), E()
+    r0.record()
+    for e0, e1, e2, e3 in ev:
+        if flush is not None:
+            flush()
         e0.record()
         buf.fwd()
         e1.record()
         if with_bwd:
+            if flush is not None:
+                flush()
+            e2.record()
             buf.bwd()
-        e2.record()
+            e3.record()
+    r1.record()
     torch.cuda.synchronize()
-    for e0, e1, e2 in ev:
-        fwd_ms.append(e0.elapsed_time(e1))
-        bwd_ms.append(e1.elapsed_time(e2))
-    return fwd_ms, bwd_ms
+    fwd_ms = [a.elapsed_time(b) for a, b, _, _ in ev]
+    bwd_ms = [c.elapsed_time(d) for _, _, c, d in ev] if with_bwd else []
+    return fwd_ms, bwd_ms, (r0.elapsed_time(r1) if flush is None else None)
 
 
 def time_step_kernel(sbuf, reps, flush):
@@ -320,27 +369,33 @@ def time_step_kernel(sbuf, reps, flush):
     return [a.elapsed_time(b) for a, b in ev]
 
 
-def workload_summary(cfg, fwd_ms, bwd_ms, peak):
-    n = cfg.elements
-    f = statistics.median(fwd_ms)
-    b = statistics.median(bwd_ms) if bwd_ms else 0.0
-    ib = io_bytes(cfg.io)
-    out = {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io,
-           "fwd_ms": f, "fwd_gbs": n * FWD_VALUES * ib / (f * 1e-3) / 1e9}
-    out["fwd_frac"] = out["fwd_gbs"] / peak
-    if not cfg.fwd_only:
-        out.update(bwd_ms=b, bwd_gbs=n * BWD_VALUES * ib / (b * 1e-3) / 1e9)
-        out["bwd_frac"] = out["bwd_gbs"] / peak
-        out["elements_per_s"] = n / ((f + b) * 1e-3)
-        out["fwd_bwd_gbs"] = n * (FWD_VALUES + BWD_VALUES) * ib / ((f + b) * 1e-3) / 1e9
-        out["fwd_bwd_frac"] = out["fwd_bwd_gbs"] / peak
+def call_roofline(kernel: str, alg_bytes: float, ms: float, peak: float, peak_kind: str, traffic):
+    """Roofline block of one C-ABI call: algorithmic bytes over its mean
+    event-timed duration, against the measured copy bandwidth."""
+    gbs = alg_bytes / (ms * 1e-3) / 1e9
+    return {"bound": "hbm", "kernel": kernel, "achieved": gbs, "peak": peak, "peak_kind": peak_kind,
+            "unit": "GB/s", "frac": gbs / peak, "traffic": traffic, "algorithmic_bytes": alg_bytes,
+            "us": ms * 1e3}
+
+
+def workload_rooflines(cfg, fwd_ms, bwd_ms, peak, peak_kind, tag):
+    """Per-call rooflines (mean times) and the fwd+bwd fraction of a workload."""
+    n, ib = cfg.elements, io_bytes(cfg.io)
+    fk, bk, _, _ = scan_kernels(cfg)
+    f = sum(fwd_ms) / len(fwd_ms)
+    out = {"workload": cfg.name,
+           "fwd": call_roofline(fk, n * FWD_VALUES * ib, f, peak, peak_kind, ncu_traffic(fk, tag))}
+    if bwd_ms:
+        b = sum(bwd_ms) / len(bwd_ms)
+        out["bwd"] = call_roofline(bk, n * BWD_VALUES * ib, b, peak, peak_kind, ncu_traffic(bk, tag))
+        gbs = n * (FWD_VALUES + BWD_VALUES) * ib / ((f + b) * 1e-3) / 1e9
+        out.update(elements_per_s=n / ((f + b) * 1e-3), fwd_bwd_gbs=gbs, fwd_bwd_frac=gbs / peak)
     else:
         out["elements_per_s"] = n / (f * 1e-3)
     return out
 
 
 def run_ours(args):
-    import numpy as np
     import torch
     rank, world, local = dist_env()
     if world > 1:
@@ -352,11 +407,11 @@ def run_ours(args):
     dev = torch.device("cuda", torch.cuda.current_device())
 
     from paper_2406_12580_gb300 import inputs as I
-    from paper_2406_12580_gb300.device import ScanBuffers, StepBuffers, to_device
+    from paper_2406_12580_gb300.device import ScanBuffers
 
     peak, peak_kind = measured_peaks()
     props = torch.cuda.get_device_properties(dev)
-    l2 = int(getattr(props, "L2_cache_size", 126 * 2**20) or 126 * 2**20)
+    l2 = int(getattr(props, "L2_cache_size", 0) or 0) or nominal_l2_bytes()
     flush_buf = torch.empty(2 * l2 // 4 + 1024, dtype=torch.float32, device=dev)
     flush = lambda: flush_buf.fill_(1.0)  # noqa: E731
 
@@ -369,10 +424,16 @@ def run_ours(args):
     inp = I.make_scan_inputs(cfg)
     buf = ScanBuffers.from_inputs(inp, device=dev)
     n = cfg.elements
+    do_flush, l2_note = l2_policy(cfg, l2)
+    tflush = flush if do_flush else None
 
     def step():
+        if tflush is not None:
+            tflush()
         buf.fwd()
         if not cfg.fwd_only:
+            if tflush is not None:
+                tflush()
             buf.bwd()
 
     for _ in range(max(3, args.warmup)):
@@ -391,7 +452,6 @@ def run_ours(args):
     preroll = 0
     while time.time() - t_pre < 0.5:
         for _ in range(20):
-            flush()
             step()
         preroll += 20
         torch.cuda.synchronize()
@@ -400,33 +460,23 @@ def run_ours(args):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
-    fwd_ms, bwd_ms = time_scan(buf, args.steps, flush, with_bwd=not cfg.fwd_only)
+    fwd_ms, bwd_ms, region_ms = time_calls(buf, args.steps, tflush, with_bwd=not cfg.fwd_only)
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     wall = time.perf_counter() - wall0
     clock_rows = sampler.stop()
 
-    total_ms = sum(fwd_ms) + sum(bwd_ms)
+    total_ms = region_ms if region_ms is not None else sum(fwd_ms) + sum(bwd_ms)
     t_max_ms = max_over_ranks(total_ms, world, device=dev)
     value = world * n * args.steps / (t_max_ms * 1e-3)
-    summ = workload_summary(cfg, fwd_ms, bwd_ms, peak)
-
-    # dominant kernel of the step and its roofline
-    favg = sum(fwd_ms) / len(fwd_ms)
-    bavg = sum(bwd_ms) / len(bwd_ms) if bwd_ms and not cfg.fwd_only else 0.0
+    tag = f"config{args.config}" if args.seq_len == 0 and not args.io else None
+    rl = workload_rooflines(cfg, fwd_ms, bwd_ms, peak, peak_kind, tag)
+    dominant = rl["bwd"] if "bwd" in rl and rl["bwd"]["us"] > rl["fwd"]["us"] else rl["fwd"]
+    _, _, kf, kb = scan_kernels(cfg)
     ib = io_bytes(cfg.io)
-    fwd_kernel, bwd_kernel, per_call, bracket = scan_kernels(cfg)
-    if bavg > favg:
-        kname, avg_ms, alg = bwd_kernel, bavg, n * BWD_VALUES * ib
-    else:
-        kname, avg_ms, alg = fwd_kernel, favg, n * FWD_VALUES * ib
-    achieved = alg / (avg_ms * 1e-3) / 1e9
-    timing = f"CUDA events around each C-ABI call ({bracket})"
-    roofline = {"bound": "hbm", "kernel": kname, "achieved": achieved, "peak": peak,
-                "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                "traffic": ncu_traffic(kname, f"config{args.config}"),
-                "algorithmic_bytes_per_launch": alg, "timing": timing}
+    step_gbs = n * ((FWD_VALUES + (0 if cfg.fwd_only else BWD_VALUES)) * ib) * args.steps / (
+        total_ms * 1e-3) / 1e9
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -434,17 +484,16 @@ def run_ours(args):
         "ms_per_step": t_max_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f32" if cfg.io == "f32" else "bf16", "data": "synthetic",
-        "config": {"workload": cfg.name, "B": cfg.B, "L": cfg.L, "D": cfg.D, "io": cfg.io,
-                   "state": "f32", "parallelism": f"replicas{world}" if world > 1 else "single",
-                   "l2": f"flushed before every timed step ({2 * l2 >> 20} MiB write)",
-                   "inputs": "seeded synthetic (paper_2406_12580_gb300.inputs), resident in HBM"},
-        "hbm_gbs": summ.get("fwd_bwd_gbs", summ["fwd_gbs"]),
-        "hbm_frac": summ.get("fwd_bwd_frac", summ["fwd_frac"]),
-        "hbm_frac_nominal": summ.get("fwd_bwd_gbs", summ["fwd_gbs"]) / NOMINAL_HBM_GBS,
-        "roofline": roofline,
-        "gpu_launches": (1 if cfg.fwd_only else 2) * per_call * args.steps,
+        "config": config_dict(cfg, world, l2_note),
+        "hbm_gbs": step_gbs, "hbm_frac": step_gbs / peak, "hbm_frac_nominal": step_gbs / NOMINAL_HBM_GBS,
+        "roofline": dominant,
+        "calls": {k: rl[k] for k in ("fwd", "bwd") if k in rl},
+        "gpu_launches": (kf + (0 if cfg.fwd_only else kb)) * args.steps,
         "wall_s_timed_region": wall,
-        "per_kernel": summ,
+        "timing": ("CUDA events on the launching stream: the K steps back to back between two "
+                   "events (value), and each C-ABI call between its own (per-call rooflines)"
+                   if region_ms is not None else
+                   "CUDA events around each C-ABI call, L2 flushed before each (value and rooflines)"),
     }
 
     rows_summary = ClockSampler.summary(clock_rows)
@@ -455,23 +504,47 @@ def run_ours(args):
     if rank == 0 and not args.quick:
         # end to end through the public API: pinned host inputs -> HBM, fwd,
         # bwd, results -> pinned host, every step
-        line["e2e"] = e2e_pipelined(inp, min(args.steps, 40), world, dev)
-        line["e2e_one_step_at_a_time"] = e2e(buf, inp, min(args.steps, 20), world)
-        line["other_workloads"] = other_workloads(flush, peak, dev, args.config)
+        del buf
+        torch.cuda.empty_cache()
+        line["e2e"] = e2e_pipelined(inp, min(args.steps, 20), world, dev)
+        configs = other_workloads(flush, peak, peak_kind, dev, args.config)
+    else:
+        configs = None
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, threads, reps, secs = cpu_oracle_rate(inp)
-        rate1, _, reps1, secs1 = cpu_oracle_rate(inp, target_s=3.0, threads=1)
-        line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
-                                "sample": f"{reps} x fwd+bwd of the whole workload "
-                                          f"({n} elements) in {secs:.1f} s, float64",
-                                "single_thread": {"value": rate1, "unit": UNIT, "cores": 1,
-                                                  "sample": f"{reps1} x fwd+bwd in {secs1:.1f} s"}}
+        line["cpu_baseline"] = cpu_baseline(cfg)
+    if configs is not None:
+        line["configs"] = configs  # last, so that a kept tail of the line holds it
     if rank == 0:
         print(json.dumps(line), flush=True)
+        if args.extras:
+            print(json.dumps({"extras": extra_workloads(flush, peak, dev)}), file=sys.stderr,
+                  flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0
+
+
+def cpu_baseline(cfg, target_s: float = 10.0):
+    """The float64 oracle, as it stands, on the host cores, over a bounded
+    sample of the workload (whole batch rows, about a second a repetition),
+    repeated for about `target_s` seconds; and on one thread."""
+    from paper_2406_12580_gb300 import inputs as I
+    rows = 1 if cfg.L * cfg.D > (1 << 20) else cfg.B
+    sample = I.make_scan_inputs(I.scaled(cfg, B=rows))
+    rate, threads, reps, secs = cpu_oracle_rate(sample, target_s=target_s)
+    if rows < cfg.B:  # grow the sample towards about a second a repetition
+        per = secs / reps
+        rows2 = int(max(1, min(cfg.B, rows / max(per, 1e-9))))
+        if rows2 > rows:
+            sample = I.make_scan_inputs(I.scaled(cfg, B=rows2))
+            rate, threads, reps, secs = cpu_oracle_rate(sample, target_s=target_s)
+    rate1, _, reps1, secs1 = cpu_oracle_rate(sample, target_s=3.0, threads=1)
+    return {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{reps} x fwd+bwd of {sample.cfg.B} of {cfg.B} batch rows "
+                      f"({sample.cfg.elements} elements) in {secs:.1f} s, float64",
+            "single_thread": {"value": rate1, "unit": UNIT, "cores": 1,
+                              "sample": f"{reps1} x fwd+bwd in {secs1:.1f} s"}}
 
 
 def e2e_pipelined(inp, reps, world, dev, nsets=3):
@@ -539,43 +612,9 @@ def e2e_pipelined(inp, reps, world, dev, nsets=3):
                            "copies in")}
 
 
-def e2e(buf, inp, reps, world):
-    """Same metric through the C ABI with host buffers: every step copies the
-    inputs from pinned host memory and reads every output back, one step at a
-    time (nothing overlaps)."""
-    import torch
-    from paper_2406_12580_gb300.device import to_device
-    cfg = inp.cfg
-    pin = lambda name: to_device(inp.io_array(name), cfg.io, "cpu", pin=False).pin_memory()  # noqa: E731
-    hx, hgl, hdh = pin("x"), pin("gl"), pin("dh") if not cfg.fwd_only else None
-    outs = [buf.h, buf.h_last] + ([] if cfg.fwd_only else [buf.dx, buf.dgl, buf.dlam])
-    host_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
-    h2d = sum(t.numel() * t.element_size() for t in (hx, hgl, hdh) if t is not None)
-    d2h = sum(t.numel() * t.element_size() for t in host_outs)
-    times = []
-    for k in range(reps + 3):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        buf.x.copy_(hx, non_blocking=True)
-        buf.gl.copy_(hgl, non_blocking=True)
-        if hdh is not None:
-            buf.dh.copy_(hdh, non_blocking=True)
-        buf.fwd()
-        if not cfg.fwd_only:
-            buf.bwd()
-        for d, s in zip(host_outs, outs):
-            d.copy_(s, non_blocking=True)
-        e1.record()
-        torch.cuda.synchronize()
-        if k >= 3:
-            times.append(e0.elapsed_time(e1))
-    ms = statistics.median(times)
-    return {"value": world * cfg.elements / (ms * 1e-3), "unit": UNIT, "ms_per_step": ms,
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
-
-
-def other_workloads(flush, peak, dev, headline):
-    """The other benchmark workloads (fewer repetitions; the same timing)."""
+def other_workloads(flush, peak, peak_kind, dev, headline):
+    """The other workloads (parity-test shapes beside the headline), each with
+    per-call rooflines; L2 flushed before every call; and the recurrent step."""
     import torch
     from paper_2406_12580_gb300 import inputs as I
     from paper_2406_12580_gb300.device import ScanBuffers, StepBuffers
@@ -586,22 +625,43 @@ def other_workloads(flush, peak, dev, headline):
         cfg = I.CONFIGS[k]
         inp = I.make_scan_inputs(cfg)
         buf = ScanBuffers.from_inputs(inp, device=dev)
-        time_scan(buf, 3, flush, with_bwd=not cfg.fwd_only)
-        f, b = time_scan(buf, 10, flush, with_bwd=not cfg.fwd_only)
-        out[f"config{k}"] = workload_summary(cfg, f, b, peak)
+        time_calls(buf, 3, flush, with_bwd=not cfg.fwd_only)
+        f, b, _ = time_calls(buf, 30, flush, with_bwd=not cfg.fwd_only)
+        out[f"config{k}"] = compact(workload_rooflines(cfg, f, b, peak, peak_kind, f"config{k}"))
         del buf, inp
         torch.cuda.empty_cache()
     for io in ("f32", "bf16"):
         scfg = I.StepConfig(f"recurrent step B=65536 D=64 {io}", 65536, 64, io, seed=4)
         sbuf = StepBuffers.from_inputs(I.make_step_inputs(scfg), device=dev)
         time_step_kernel(sbuf, 3, flush)
-        ms = statistics.median(time_step_kernel(sbuf, 20, flush))
-        gbs = scfg.elements * step_bytes_per_elem(io) / (ms * 1e-3) / 1e9
-        out[f"step_{io}"] = {"workload": scfg.name, "ms": ms,
-                             "elements_per_s": scfg.elements / (ms * 1e-3), "gbs": gbs,
-                             "frac": gbs / peak}
+        ms = sum(time_step_kernel(sbuf, 30, flush)) / 30
+        r = call_roofline("step_kernel", scfg.elements * step_bytes_per_elem(io), ms, peak,
+                          peak_kind, None)
+        out[f"step_{io}"] = {"us": round(r["us"], 2), "frac": round(r["frac"], 3)}
         del sbuf
-    out["step_f32_graph"] = step_graph(flush, peak, dev)
+    g = step_graph(flush, peak, dev)
+    out["step_f32_graph8"] = {"us": round(g["ms_per_step"] * 1e3, 2), "frac": round(g["frac"], 3)}
+    return out
+
+
+def compact(rl):
+    """A workload's rooflines, short enough for the end of the JSON line: per
+    call the mean event-timed microseconds, fraction of the measured copy
+    bandwidth and ncu DRAM bytes per launch (null if not captured on these
+    kernel sources); and the fwd+bwd fraction."""
+    out = {}
+    for k in ("fwd", "bwd"):
+        if k in rl:
+            out[k] = {"kernel": rl[k]["kernel"], "us": round(rl[k]["us"], 2),
+                      "frac": round(rl[k]["frac"], 3), "traffic": rl[k]["traffic"]}
+    if "fwd_bwd_frac" in rl:
+        out["frac"] = round(rl["fwd_bwd_frac"], 3)
+    return out
+
+
+def extra_workloads(flush, peak, dev):
+    """Workloads beyond the scope table's configurations (--extras)."""
+    out = {}
     for io in ("f32", "bf16"):
         out[f"steps_k8_{io}"] = steps_workload(io, flush, peak, dev)
     for k in (1, 2):

@@ -25,7 +25,9 @@ def test_reference_arm_prints_one_contract_line():
         assert key in d, key
     assert d["steps"] == 1 and d["warmup"] >= 3 and d["n_gpus"] == 1
     assert d["value"] > 0 and d["higher_is_better"] is True
-    assert d["config"]["workload"] and d["config"]["B"] == 256
+    # the headline workload, with the same config keys as the GPU arm's line
+    assert d["config"]["workload"] and (d["config"]["B"], d["config"]["L"], d["config"]["D"]) == (8, 32768, 512)
+    assert set(d["config"]) == {"workload", "B", "L", "D", "io", "state", "parallelism", "l2", "inputs"}
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     e2e = d["e2e"]
