@@ -316,15 +316,20 @@ BLR_API const char* blr_last_error_string(void);
  * the library and kept until the process exits. It never calls an allocator.
  *  - Problems whose workspace (blr_workspace_bytes) exceeds 128 MiB return
  *    BLR_ERR_UNSUPPORTED with nothing enqueued; use blr_scan_fwd for them.
- *  - The first call on each device looks up the scratch array's device
- *    address (cudaGetSymbolAddress); make that first call before any stream
- *    capture that includes it.
+ *  - The first call on each device (and the first after the device's CUDA
+ *    context has been reset or re-created) looks up the scratch array's
+ *    device address (cudaGetSymbolAddress); make that first call before any
+ *    stream capture that includes it.
  *  - All calls on a device share the one scratch array, and each call reuses
  *    whatever the last one left there after clearing what must start empty.
- *    Calls that may overlap on the GPU (different streams without ordering
- *    between them) race on it: serialise them.
- *  - The scratch cannot be passed to blr_scan_bwd or blr_workspace_status:
- *    this is a forward-only (inference) path.
+ *    The backward entry points called with ws == NULL use the same array
+ *    (they recompute the forward's carries in it). Calls of either kind that
+ *    may overlap on the GPU (different streams without ordering between
+ *    them) race on it: serialise them.
+ *  - blr_workspace_status with ws == NULL reads the array's error word. The
+ *    array is not a workspace a caller can name: a backward that should use
+ *    this forward's carries cannot be given them (with ws == NULL it
+ *    recomputes them), so this is in effect a forward-only (inference) path.
  */
 BLR_API blr_status blr_scan_fwd_noalloc(const blr_desc* desc, const void* x, const void* gate_logits,
                                         const float* lambda, const float* h0, void* h,

@@ -947,30 +947,53 @@ const char* blr_last_error_string(void) { return g_last_error; }
 // kLibraryScratchBytes, present on every GPU that loads this library until
 // the process exits. The host never dereferences the array's name (in host
 // code it is only a stand-in for the device symbol); the device address comes
-// from cudaGetSymbolAddress, once per device.
+// from cudaGetSymbolAddress, looked up once per device and context.
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kLibraryScratchBytes];
 
 namespace {
 
 constexpr int kMaxDevices = 64;
 
-__device__ __align__(256) unsigned char g_noalloc_scratch[kLibraryScratchBytes];
-
 std::mutex g_scratch_mutex;
 void* g_scratch_ptr[kMaxDevices] = {};
+CUcontext g_scratch_ctx[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device (set up on the
-// first call on each device).
+// The calling thread's current CUDA context (NULL if none), through the
+// runtime's driver entry point (the library links only the CUDA runtime).
+CUcontext current_context() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(ptr);
+  });
+  CUcontext ctx = nullptr;
+  if (fn == nullptr || fn(&ctx) != CUDA_SUCCESS) return nullptr;
+  return ctx;
+}
+
+// Device address of the scratch array on the current device, set up on the
+// first call on each device and again whenever the device's context has
+// changed since (a reset or a re-created primary context loads the module
+// anew, so an address from before would be stale).
 blr_status noalloc_scratch(void** out) {
   int dev = 0;
   BLR_TRY(cuda_check(cudaGetDevice(&dev), "cudaGetDevice"));
   if (dev < 0 || dev >= kMaxDevices)
     return fail(BLR_ERR_UNSUPPORTED, "device index %d above the scratch table", dev);
   std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (g_scratch_ptr[dev] == nullptr) {
+  CUcontext ctx = current_context();
+  if (g_scratch_ptr[dev] == nullptr || ctx == nullptr || ctx != g_scratch_ctx[dev]) {
     void* p = nullptr;
     BLR_TRY(cuda_check(cudaGetSymbolAddress(&p, g_noalloc_scratch),
                        "cudaGetSymbolAddress of the static scratch"));
     g_scratch_ptr[dev] = p;
+    g_scratch_ctx[dev] = current_context();  // current now, if it was not before the lookup
   }
   *out = g_scratch_ptr[dev];
   return BLR_OK;

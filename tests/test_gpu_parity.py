@@ -8,8 +8,8 @@ bfloat16 I/O.
 import numpy as np
 import pytest
 
-from gpu_common import (TOL, compare, gpu_outputs, gpu_scan, gpu_scan_gated, gpu_step, normwise,
-                        oracle_outputs)
+from gpu_common import (TOL, compare, compare_by_rows, gpu_outputs, gpu_scan, gpu_scan_gated,
+                        gpu_step, normwise, oracle_outputs)
 from paper_2406_12580_gb300 import inputs as I
 
 torch = pytest.importorskip("torch")
@@ -79,13 +79,12 @@ def _sampled_channels(D):
 
 
 @pytest.mark.parametrize("k", [3, 4])
-def test_config_full_size_sampled(k):
-    """Configurations 3-4 at full size; the oracle runs the sampled channels in
-    full (every batch row and step of each: the recurrence is per channel)."""
+def test_config_full_size_every_channel(k):
+    """Configurations 3-4 at full size against the oracle on every batch row
+    and channel, a few batch rows at a time (which bounds host memory)."""
     inp = I.make_scan_inputs(I.CONFIGS[k])
     buf = gpu_scan(inp)
-    dsel = _sampled_channels(inp.cfg.D)
-    errs = compare(inp, gpu_outputs(buf, dsel), oracle_outputs(inp, dsel, threads=0))
+    errs = compare_by_rows(inp, buf, rows=1 if k == 4 else 8)
     print(f"config {k}: {errs}")
 
 
@@ -659,8 +658,9 @@ def test_graph_capture_replays_eager(io, shape):
     # the same kernels, so the same values up to the order of float atomics
     # (dLambda) and of look-back combines: a look-back folds whichever
     # predecessors have published when it reads, so float32 carries may differ
-    # in their last bits between calls, and a bfloat16 output by one rounding
-    # step (2^-8 of its magnitude) where such a carry sits at a rounding boundary
-    tol = 1e-6 if io == I.F32 else 2.0 ** -8
+    # in their last bits between calls, and a bfloat16 output by one unit in
+    # its last place (at most 2^-7 of its magnitude) where such a carry sits at
+    # a rounding boundary
+    tol = 1e-6 if io == I.F32 else 2.0 ** -7
     for k in eager:
         assert normwise(got[k], eager[k]) <= tol, k
