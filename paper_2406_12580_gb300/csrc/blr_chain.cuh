@@ -14,24 +14,30 @@
 //   compute (kChainWarps warps, a slice of kChainSlice steps each): pass A of
 //      tile n evaluates the gates of Sec. 3.2 for the slice from the stage
 //      (which is then released), folds it serially from a zero state (hl_t,
-//      and ap_t = the product of the alphas so far, so that h_t = hl_t +
-//      ap_t h_start, both kept in registers) and publishes the slice's map.
+//      and am_t = the product of the alphas so far minus one, so that h_t =
+//      hl_t + (1 + am_t) h_start) and publishes the slice's map (A - 1, U).
 //      Then pass C of tile n - kChainLag, whose entering states the scanners
-//      have found meanwhile: h_t = hl_t + ap_t h_start is written to global
+//      have found meanwhile: h_t = hl_t + (1 + am_t) h_start is written to global
 //      memory from registers (coalesced 128-byte rows), with the kept states
 //      the backward starts from;
 //   scanners (kChainScanners warps, tiles in turn): compose the slice maps into the
-//      tile's map (A, U) (the operator of Sec. 3.3, (a2, u2) . (a1, u1) =
-//      (a2 a1, a2 u1 + u2)), publish it, find the state entering the tile with
+//      tile's map (the operator of Sec. 3.3, (a2, u2) . (a1, u1) = (a2 a1,
+//      a2 u1 + u2)), publish it, find the state entering the tile with
 //      a decoupled look-back over the records of the tiles before it in the
 //      same chain, publish the state after the tile, and hand every slice its
 //      starting state.
 // The look-back's round trips to L2 thus overlap kChainLag tiles' arithmetic
 // instead of stalling it, and the ring keeps several tiles' loads in flight.
 //
+// Products of alphas are carried as their difference from one (m = A - 1):
+// with slow decays a product of a few alphas lies within 1e-3 of one, where a
+// float32 holds only a few significant digits of 1 - A, which the large states
+// of slow decays then multiply. A map h -> A h + U is applied as
+// (m h + h) + U, and two maps compose as m = m1 + m2 + m1 m2.
+//
 // Records validate themselves: a record is one relaxed 32- or 64-bit store of
 // a value that is never the all-ones pattern the records are filled with
-// before the call (A lies in [0, 1]; a float state is never that NaN).
+// before the call (A - 1 lies in (-1, 0]; a float state is never that NaN).
 #pragma once
 
 #include "blr_seq.cuh"
@@ -90,14 +96,22 @@ struct ChainSmem {
                 tmem % 16 == 0 && bars % 16 == 0, "");
 };
 
+// The map h -> (1 + m) h + U applied to h, and the composition of the minus-one
+// parts of two maps' products.
+__device__ __forceinline__ float map_apply(float m, float h, float U) { return fmaf(m, h, h) + U; }
+__device__ __forceinline__ float2 map_apply2(float2 m, float2 h, float2 U) {
+  return __fadd2_rn(__ffma2_rn(m, h, h), U);
+}
+__device__ __forceinline__ float m_compose(float m1, float m2) { return fmaf(m1, m2, m1 + m2); }
+
 // Pass A for one lane: the gates of the TS rows of its warp's slice (as the
 // serial forward evaluates them), then the slice folded from a zero state.
-// On return hl[s] is the state after row s from a zero start and ap[s] the
-// product of the alphas of rows 0 .. s.
+// On return hl[s] is the state after row s from a zero start and am[s] the
+// product of the alphas of rows 0 .. s minus one.
 template <class IO, class G, bool POLY, int TS>
 __device__ __forceinline__ void chain_fold(const unsigned char* lb, const float (&k)[IO::VEC],
                                            const float (&kh)[IO::VEC], float (&hl)[TS][IO::VEC],
-                                           float (&ap)[TS][IO::VEC]) {
+                                           float (&am)[TS][IO::VEC]) {
   using Raw = typename IO::Raw;
   constexpr int V = IO::VEC;
   constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
@@ -112,7 +126,7 @@ __device__ __forceinline__ void chain_fold(const unsigned char* lb, const float 
 #pragma unroll
       for (int v = 0; v < V; ++v) {
         const float e = expm1_neg<G::kDeg, POLY>(G::decay_log_half(rv[v], kh[v]));
-        ap[s][v] = 1.0f + e;
+        am[s][v] = e;
         hl[s][v] = G::sqrt(-e * (e + 2.0f)) * G::gated_x_half(iv[v], xv[v]);
       }
     } else {
@@ -122,20 +136,21 @@ __device__ __forceinline__ void chain_fold(const unsigned char* lb, const float 
 #pragma unroll
       for (int v = 0; v < V; ++v) {
         const float e = expm1_neg<G::kDeg, POLY>(G::decay_log(rv[v], k[v], kh[v]));
-        ap[s][v] = 1.0f + e;
+        am[s][v] = e;
         hl[s][v] = G::sqrt(-e * (e + 2.0f)) * (G::sigmoid(iv[v]) * xv[v]);
       }
     }
   }
 #pragma unroll
   for (int v = 0; v < V; ++v) {
-    float H = 0.0f, A = 1.0f;
+    float H = 0.0f, m = 0.0f;
 #pragma unroll
     for (int s = 0; s < TS; ++s) {
-      H = fmaf(ap[s][v], H, hl[s][v]);
-      A *= ap[s][v];
+      const float e = am[s][v], alpha = 1.0f + e;
+      H = fmaf(alpha, H, hl[s][v]);
+      m = fmaf(alpha, m, e);  // alpha (1 + m) - 1
       hl[s][v] = H;
-      ap[s][v] = A;
+      am[s][v] = m;
     }
   }
 }
@@ -145,7 +160,7 @@ __device__ __forceinline__ void chain_fold(const unsigned char* lb, const float 
 // as chain_fold with GatesFast.
 template <bool POLY, int TS>
 __device__ __forceinline__ void chain_fold_bf16x2(const unsigned char* lb, float2 kh,
-                                                  float2 (&hl)[TS], float2 (&ap)[TS]) {
+                                                  float2 (&hl)[TS], float2 (&am)[TS]) {
   using IO = Io<__nv_bfloat16, 2>;
   constexpr uint32_t ROWB = 128;
   constexpr uint32_t BOX = kChainTile * ROWB;
@@ -167,7 +182,7 @@ __device__ __forceinline__ void chain_fold_bf16x2(const unsigned char* lb, float
     } else {
       e = make_float2(expm1_neg<4, false>(l.x), expm1_neg<4, false>(l.y));
     }
-    ap[s] = __fadd2_rn(one, e);
+    am[s] = e;
     // 1 - alpha^2 = -e (e + 2); u = sqrt(1 - alpha^2) i x with i x = (x/2) tanh(iota/2) + x/2
     const float2 m = __fmul2_rn(e, __fadd2_rn(e, two));
     const float2 gx = __ffma2_rn(make_float2(xv[0], xv[1]),
@@ -175,13 +190,14 @@ __device__ __forceinline__ void chain_fold_bf16x2(const unsigned char* lb, float
                                  make_float2(xv[0], xv[1]));
     hl[s] = __fmul2_rn(make_float2(sqrt_approx(-m.x), sqrt_approx(-m.y)), gx);
   }
-  float2 H = make_float2(0.0f, 0.0f), A = one;
+  float2 H = make_float2(0.0f, 0.0f), m = make_float2(0.0f, 0.0f);
 #pragma unroll
   for (int s = 0; s < TS; ++s) {
-    H = __ffma2_rn(ap[s], H, hl[s]);
-    A = __fmul2_rn(A, ap[s]);
+    const float2 alpha = __fadd2_rn(one, am[s]);
+    H = __ffma2_rn(alpha, H, hl[s]);
+    m = __ffma2_rn(alpha, m, am[s]);  // alpha (1 + m) - 1
     hl[s] = H;
-    ap[s] = A;
+    am[s] = m;
   }
 }
 
@@ -215,21 +231,21 @@ __device__ __forceinline__ void chain_window_load(const unsigned long long* agg,
 // it returns what it has.
 __device__ __forceinline__ float chain_walk(const unsigned long long* agg, const uint32_t* inc,
                                            int64_t BD, int64_t j, uint32_t* err, ChainWindow& w) {
-  float ea = 1.0f, eu = 0.0f;  // the fold of the aggregates walked so far
+  float em = 0.0f, eu = 0.0f;  // the fold of the aggregates walked so far: h -> (1 + em) h + eu
   for (;;) {
     int adv = kChainWindow;
     bool open = true, wait = false;
 #pragma unroll
     for (int q = 0; q < kChainWindow; ++q) {
       if (open) {
-        if (w.in[q] != kEmpty) return fmaf(ea, __uint_as_float(w.in[q]), eu);
+        if (w.in[q] != kEmpty) return map_apply(em, __uint_as_float(w.in[q]), eu);
         if (agg_empty(w.ag[q])) {  // nothing published yet: wait for it, then re-read from it
           open = false;
           wait = true;
           adv = q;
         } else {
-          eu = fmaf(ea, __uint_as_float((uint32_t)(w.ag[q] >> 32)), eu);
-          ea *= __uint_as_float((uint32_t)w.ag[q]);
+          eu = map_apply(em, __uint_as_float((uint32_t)(w.ag[q] >> 32)), eu);
+          em = m_compose(em, __uint_as_float((uint32_t)w.ag[q]));
         }
       }
     }
@@ -360,16 +376,16 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
       const int64_t d0 = (int64_t)c.z * CHW + lane * VEC;
       const bool ch_ok = d0 < p.D;
       mbar_wait(&maps_ready[m], (uint32_t)(n / MS) & 1u, err);
-      float TA[VEC], TU[VEC], hs[VEC];
+      float TM[VEC], TU[VEC], hs[VEC];  // the tile's map h -> (1 + TM) h + TU
 #pragma unroll
       for (int v = 0; v < VEC; ++v) {
-        TA[v] = 1.0f;
+        TM[v] = 0.0f;
         TU[v] = 0.0f;
 #pragma unroll
         for (int w = 0; w < NW; ++w) {
           const float2 e = maps[(m * NW + w) * CHW + lane * VEC + v];
-          TU[v] = fmaf(e.x, TU[v], e.y);
-          TA[v] *= e.x;
+          TU[v] = map_apply(e.x, TU[v], e.y);
+          TM[v] = m_compose(TM[v], e.x);
         }
         hs[v] = 0.0f;
       }
@@ -383,7 +399,7 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
           }
         } else {
 #pragma unroll
-          for (int v = 0; v < VEC; ++v) st_record(&agg[rec + v], pack_agg(TA[v], TU[v]));
+          for (int v = 0; v < VEC; ++v) st_record(&agg[rec + v], pack_agg(TM[v], TU[v]));
           ChainWindow win[VEC];
 #pragma unroll
           for (int v = 0; v < VEC; ++v)
@@ -393,7 +409,7 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
             hs[v] = chain_walk(agg + ch0 + v, inc + ch0 + v, BD, c.x - 1, err, win[v]);
         }
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) st_record(&inc[rec + v], __float_as_uint(fmaf(TA[v], hs[v], TU[v])));
+        for (int v = 0; v < VEC; ++v) st_record(&inc[rec + v], __float_as_uint(map_apply(TM[v], hs[v], TU[v])));
       }
       // every slice's starting state: the carry through the slices before it,
       // written over the slice's map
@@ -404,7 +420,7 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
           float2* e = &maps[(m * NW + w) * CHW + lane * VEC + v];
           const float2 mw = *e;
           e->x = hs[v];
-          hs[v] = fmaf(mw.x, hs[v], mw.y);
+          hs[v] = map_apply(mw.x, hs[v], mw.y);
         }
       }
       if (lane == 0) meta[m] = c;
@@ -448,14 +464,14 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
 #pragma unroll
         for (int r = 0; r < TS; ++r) {
           if constexpr (BF16X2) {
-            const float2 o = __ffma2_rn(make_float2(park[4 * r + 1], park[4 * r + 3]), make_float2(hs[0], hs[1]),
-                                        make_float2(park[4 * r], park[4 * r + 2]));
+            const float2 o = map_apply2(make_float2(park[4 * r + 1], park[4 * r + 3]),
+                                        make_float2(hs[0], hs[1]), make_float2(park[4 * r], park[4 * r + 2]));
             out[r][0] = o.x;
             out[r][1] = o.y;
           } else {
 #pragma unroll
             for (int v = 0; v < VEC; ++v)
-              out[r][v] = fmaf(park[2 * (r * VEC + v) + 1], hs[v], park[2 * (r * VEC + v)]);
+              out[r][v] = map_apply(park[2 * (r * VEC + v) + 1], hs[v], park[2 * (r * VEC + v)]);
           }
         }
         const uint32_t d0 = (uint32_t)c.z * CHW + lane * VEC;  // D < 2^24
@@ -504,20 +520,20 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         if constexpr (BF16X2) {
           const float2 r0 = rates[s * CHW + lane * 2], r1 = rates[s * CHW + lane * 2 + 1];
           const float2 kh = make_float2(r0.y, r1.y);
-          float2 hl[TS], ap[TS];
+          float2 hl[TS], am[TS];
           if (polys[s])
-            chain_fold_bf16x2<true, TS>(lb, kh, hl, ap);
+            chain_fold_bf16x2<true, TS>(lb, kh, hl, am);
           else
-            chain_fold_bf16x2<false, TS>(lb, kh, hl, ap);
+            chain_fold_bf16x2<false, TS>(lb, kh, hl, am);
 #pragma unroll
           for (int r = 0; r < TS; ++r) {
             park[4 * r] = hl[r].x;
-            park[4 * r + 1] = ap[r].x;
+            park[4 * r + 1] = am[r].x;
             park[4 * r + 2] = hl[r].y;
-            park[4 * r + 3] = ap[r].y;
+            park[4 * r + 3] = am[r].y;
           }
-          mapv[0] = make_float2(ap[TS - 1].x, hl[TS - 1].x);
-          mapv[1] = make_float2(ap[TS - 1].y, hl[TS - 1].y);
+          mapv[0] = make_float2(am[TS - 1].x, hl[TS - 1].x);
+          mapv[1] = make_float2(am[TS - 1].y, hl[TS - 1].y);
         } else {
           float k[VEC], kh[VEC];
 #pragma unroll
@@ -526,11 +542,11 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
             k[v] = r.x;
             kh[v] = r.y;
           }
-          float hl[TS][VEC], ap[TS][VEC];
+          float hl[TS][VEC], am[TS][VEC];
           if (polys[s])
-            chain_fold<IO, G, true, TS>(lb, k, kh, hl, ap);
+            chain_fold<IO, G, true, TS>(lb, k, kh, hl, am);
           else
-            chain_fold<IO, G, false, TS>(lb, k, kh, hl, ap);
+            chain_fold<IO, G, false, TS>(lb, k, kh, hl, am);
 #pragma unroll
           for (int i2 = 0; i2 < 16; ++i2) park[i2] = 0.0f;
 #pragma unroll
@@ -538,11 +554,11 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
 #pragma unroll
             for (int v = 0; v < VEC; ++v) {
               park[2 * (r * VEC + v)] = hl[r][v];
-              park[2 * (r * VEC + v) + 1] = ap[r][v];
+              park[2 * (r * VEC + v) + 1] = am[r][v];
             }
           }
 #pragma unroll
-          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(ap[TS - 1][v], hl[TS - 1][v]);
+          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(am[TS - 1][v], hl[TS - 1][v]);
         }
         mbar_arrive(&empty[s]);  // the stage is read: the producer may refill it
 #pragma unroll

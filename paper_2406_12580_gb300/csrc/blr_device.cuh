@@ -361,7 +361,8 @@ __device__ __forceinline__ void st_record(uint32_t* p, uint32_t v) {
 __device__ __forceinline__ void st_record(unsigned long long* p, unsigned long long v) {
   asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
-// An aggregate (A, U): A in the low word (A is in [0, 1], never the empty pattern).
+// An aggregate (A, U): A in the low word. The tiled kernels store A in [0, 1],
+// the chained forward A - 1 in (-1, 0]: a finite float, never the empty pattern.
 __device__ __forceinline__ unsigned long long pack_agg(float A, float U) {
   return (unsigned long long)__float_as_uint(A) | ((unsigned long long)__float_as_uint(U) << 32);
 }

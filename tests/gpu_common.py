@@ -14,12 +14,10 @@ from paper_2406_12580_gb300.device import ScanBuffers, StepBuffers, to_host_f64
 TOL = {I.F32: 1e-5, I.BF16: 2e-2}
 # Elementwise bounds on max |gpu - oracle| / (|oracle| + 1e-3 max|oracle|)
 # (relative per element, absolute below a thousandth of the tensor's scale):
-# measured at most 3.2e-4 (float32) and 2.4e-2 (bfloat16: one output rounding
-# of up to 2^-8 relative, plus the float32 state's error, which over the
-# 1/(1 - alpha) ~ 1e4 steps that slow decays remember reaches a few 1e-5 of the
-# row's scale, a few percent at the floor; the long-sequence workload on every
-# channel) over the whole suite.
-ELEM_TOL = {I.F32: 2e-3, I.BF16: 5e-2}
+# measured at most 3.2e-4 (float32) and 6e-3 (bfloat16: one output rounding of
+# up to 2^-8 relative, plus tanh.approx's 2^-11 in the gates) over the whole
+# suite, the long-sequence workload on every channel included.
+ELEM_TOL = {I.F32: 2e-3, I.BF16: 2e-2}
 # dLambda per channel: |gpu - oracle| / (|oracle| + 1e-6 max|oracle|), so that
 # a channel with a small gradient is checked at its own size; measured at most
 # 4.1e-4 (float32) and 3.5e-2 (bfloat16, whose per-step terms carry the
