@@ -19,9 +19,11 @@
 // uses as its starting points: the backward walks the sequence from the end in
 // sub-blocks of RB steps, recomputes the sub-block's gates and states forward
 // from the kept state (holding E = alpha - 1, 1 / sqrt(1 - alpha^2) and
-// h_{t-1} per element in registers), then runs the reverse recurrence
+// h_{t-1} per element in registers; bfloat16 lanes: alpha, sqrt(1 - alpha^2)
+// and the d l factor), then runs the reverse recurrence
 // g_t = dh_t + alpha_{t+1} g_{t+1} through it, writing dx, d rho and d iota and
-// accumulating d Lambda.
+// accumulating d Lambda. bfloat16 lanes carry their two channels as packed
+// float pairs (paired multiply-adds).
 //
 // The forward's first block also restarts the workspace bookkeeping (error
 // word, problem tag, the backward's exit counter and d Lambda partial sums), so
@@ -197,7 +199,90 @@ __device__ __forceinline__ void seg_adjoint_in(const float2* maps, int64_t BD, i
   }
 }
 
+// ------------------------------------------------- packed bfloat16 pairs
+//
+// A bfloat16 lane's two channels as one float2, so that the multiply-adds of
+// both run as one paired instruction (fma/mul/add.rn.f32x2); the
+// transcendental units (tanh, rsqrt, sqrt) stay scalar. Every paired operation
+// rounds each half exactly as its scalar counterpart would.
+
+constexpr uint32_t kBf2Half = 0x3f003f00u;     // (0.5, 0.5) as bfloat16 pairs
+constexpr uint32_t kBf2NegHalf = 0xbf00bf00u;  // (-0.5, -0.5)
+
+__device__ __forceinline__ float2 f2(float a) { return make_float2(a, a); }
+// The pair t as floats.
+__device__ __forceinline__ float2 bf2_unpack(uint32_t t) {
+  return make_float2(__uint_as_float(t << 16), __uint_as_float(t & 0xffff0000u));
+}
+// The pair t times s2 (a bfloat16 pair of +-0.5: exact, a sign and exponent
+// change), as floats.
+__device__ __forceinline__ float2 bf2_scaled(uint32_t t, uint32_t s2) {
+  uint32_t u;
+  asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(u) : "r"(t), "r"(s2));
+  return bf2_unpack(u);
+}
+__device__ __forceinline__ uint32_t bf2_pack(float2 v) { return pack_bf16x2(v.x, v.y); }
+// A shared-memory word read afresh where it is used, never kept in a register
+// from an earlier read of the same word (the backward re-reads a step's inputs
+// instead of holding them, and their gates, across a sub-block).
+__device__ __forceinline__ uint32_t lds_again(const unsigned char* p) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(smem_addr(p)));
+  return v;
+}
+__device__ __forceinline__ float2 tanh2(float2 a) {
+  return make_float2(tanh_approx(a.x), tanh_approx(a.y));
+}
+// e^l - 1 for l <= 0 (GatesFast: the degree-4 series, ex2 beyond its range
+// unless POLY), as expm1_neg<4, POLY> on each half.
+template <bool POLY>
+__device__ __forceinline__ float2 expm1_neg2(float2 l) {
+  if constexpr (POLY) {
+    float2 q = __ffma2_rn(f2(1.0f / 24), l, f2(1.0f / 6));
+    q = __ffma2_rn(q, l, f2(0.5f));
+    q = __ffma2_rn(q, l, f2(1.0f));
+    return __fmul2_rn(q, l);
+  } else {
+    return make_float2(expm1_neg<4, false>(l.x), expm1_neg<4, false>(l.y));
+  }
+}
+
 // ------------------------------------------------------------------ forward
+
+// seq_fwd_stage for a bfloat16 lane under GatesFast, without the merge: the
+// same arithmetic in the same order, on packed pairs.
+template <bool POLY, bool FULL, int R, int RB>
+__device__ __forceinline__ void seq_fwd_stage_bf16x2(unsigned char* sb, int rows, float2 kh,
+                                                     float2& hc, float* carry, int64_t& cidx,
+                                                     int64_t n_carry, int64_t BD, bool ch_ok) {
+  constexpr uint32_t ROWB = 128;
+  constexpr uint32_t BOX = R * ROWB;
+  float2 al[R], uu[R];
+#pragma unroll
+  for (int s = 0; s < R; ++s) {
+    if (FULL || s < rows) {
+      const float2 hx = bf2_scaled(*reinterpret_cast<const uint32_t*>(sb + s * ROWB), kBf2Half);
+      const float2 hr = bf2_scaled(*reinterpret_cast<const uint32_t*>(sb + BOX + s * ROWB), kBf2Half);
+      const float2 hi = bf2_scaled(*reinterpret_cast<const uint32_t*>(sb + 2 * BOX + s * ROWB), kBf2Half);
+      const float2 e = expm1_neg2<POLY>(__ffma2_rn(kh, tanh2(hr), kh));  // l = kh tanh(rho/2) + kh
+      al[s] = __fadd2_rn(f2(1.0f), e);
+      const float2 m2 = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));  // -(1 - alpha^2)
+      const float2 n = make_float2(sqrt_approx(-m2.x), sqrt_approx(-m2.y));
+      uu[s] = __fmul2_rn(n, __ffma2_rn(hx, tanh2(hi), hx));  // sqrt(1 - alpha^2) i x
+    }
+  }
+#pragma unroll
+  for (int s = 0; s < R; ++s) {
+    if (FULL || s < rows) {
+      hc = __ffma2_rn(al[s], hc, uu[s]);
+      *reinterpret_cast<uint32_t*>(sb + s * ROWB) = bf2_pack(hc);
+      if ((s + 1) % RB == 0) {  // a kept state: after step (cidx + 1) RB - 1
+        if (cidx < n_carry && ch_ok) *reinterpret_cast<float2*>(carry + cidx * BD) = hc;
+        ++cidx;
+      }
+    }
+  }
+}
 
 // One stage, rows [0, rows) (all R when FULL). Phase 1 evaluates the
 // gates of every row (independent work), phase 2 runs the recurrence and
@@ -292,6 +377,8 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
   constexpr int NB = GATED ? 4 : 3;  // boxes per stage: x, rho, iota (, z)
   constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
   static_assert(R % RB == 0, "kept states must fall on stage rows");
+  // bfloat16 lanes without the merge run their arithmetic on packed pairs
+  constexpr bool kPacked = G::kHalfInputs && VEC == 2 && !GATED;
   const Plan& p = a.p;
   extern __shared__ unsigned char seq_smem[];
   SeqRing<NB, BOX> ring{align128(seq_smem), nullptr, a.stages};
@@ -359,7 +446,20 @@ __global__ void __launch_bounds__(32) seq_fwd_kernel(const __grid_constant__ Seq
     unsigned char* lb = sb + lane * VEC * sizeof(T);
     const int64_t left = len - j * R;
     const int rows = (int)(left < R ? left : R);
-    if (rows == R) {
+    if constexpr (kPacked) {
+      float2 hc2 = make_float2(hc[0], hc[1]);
+      const float2 kh2 = make_float2(kh[0], kh[1]);
+      if (rows == R) {
+        if (poly)
+          seq_fwd_stage_bf16x2<true, true, R, RB>(lb, rows, kh2, hc2, carry, cidx, n_carry, BD, ch_ok);
+        else
+          seq_fwd_stage_bf16x2<false, true, R, RB>(lb, rows, kh2, hc2, carry, cidx, n_carry, BD, ch_ok);
+      } else {
+        seq_fwd_stage_bf16x2<false, false, R, RB>(lb, rows, kh2, hc2, carry, cidx, n_carry, BD, ch_ok);
+      }
+      hc[0] = hc2.x;
+      hc[1] = hc2.y;
+    } else if (rows == R) {
       if (poly)
         seq_fwd_stage<IO, G, true, true, R, RB, GATED>(lb, rows, k, kh, hc, carry, cidx, n_carry, BD, ch_ok);
       else
@@ -465,11 +565,12 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
 #pragma unroll
         for (int v = 0; v < V; ++v) G::silu_grad(zv[v], sf[v], sdf[v]);
       }
-      IO::unpack(*reinterpret_cast<const Raw*>(s_x + s * ROWB), xv);
-      if constexpr (G::kHalfInputs) {
-        IO::unpack_half(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
-        IO::unpack_half(*reinterpret_cast<const Raw*>(s_i + s * ROWB), iv);
+      if constexpr (G::kHalfInputs) {  // bfloat16 pairs: re-read, not held from the recompute
+        IO::unpack(lds_again(s_x + s * ROWB), xv);
+        IO::unpack_half(lds_again(s_r + s * ROWB), rv);
+        IO::unpack_half(lds_again(s_i + s * ROWB), iv);
       } else {
+        IO::unpack(*reinterpret_cast<const Raw*>(s_x + s * ROWB), xv);
         IO::unpack(*reinterpret_cast<const Raw*>(s_r + s * ROWB), rv);
         IO::unpack(*reinterpret_cast<const Raw*>(s_i + s * ROWB), iv);
       }
@@ -509,6 +610,66 @@ __device__ __forceinline__ void seq_bwd_sub(unsigned char* lb, int row0, int sro
   }
 }
 
+// seq_bwd_sub for a bfloat16 lane under GatesFast, without the merge, on
+// packed pairs. The forward recompute keeps, per step, alpha, -sqrt(1 - alpha^2)
+// and c = h_{t-1} - alpha i x / sqrt(1 - alpha^2) (so that d l = alpha g c);
+// the reverse recurrence re-reads the step's inputs for i and r, and uses
+// r (1 - r) = (1 - tanh(rho/2)^2) / 4, so d rho = d l (k/4) (1 - tanh^2).
+// kq = k/4 and nkq = -k/4 per channel.
+template <bool POLY, bool FULL, int R, int RB>
+__device__ __forceinline__ void seq_bwd_sub_bf16x2(unsigned char* lb, int row0, int srows, float2 kh,
+                                                   float2 kq, float2 nkq, float2& hc, float2& w,
+                                                   float2& dlr) {
+  constexpr uint32_t ROWB = 128;
+  constexpr uint32_t BOX = R * ROWB;
+  unsigned char* s_dh = lb + row0 * ROWB;
+  const unsigned char* s_x = s_dh + BOX;
+  unsigned char* s_r = s_dh + 2 * BOX;
+  unsigned char* s_i = s_dh + 3 * BOX;
+  float2 AL[RB], NQ[RB], CP[RB];
+#pragma unroll
+  for (int s = 0; s < RB; ++s) {
+    if (FULL || s < srows) {
+      const float2 nhx = bf2_scaled(*reinterpret_cast<const uint32_t*>(s_x + s * ROWB), kBf2NegHalf);
+      const float2 hr = bf2_scaled(*reinterpret_cast<const uint32_t*>(s_r + s * ROWB), kBf2Half);
+      const float2 hi = bf2_scaled(*reinterpret_cast<const uint32_t*>(s_i + s * ROWB), kBf2Half);
+      const float2 e = expm1_neg2<POLY>(__ffma2_rn(kh, tanh2(hr), kh));
+      const float2 m2 = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));  // -(1 - alpha^2)
+      const float2 rs = make_float2(rsqrt_approx(fmaxf(-m2.x, 1e-30f)), rsqrt_approx(fmaxf(-m2.y, 1e-30f)));
+      const float2 al = __fadd2_rn(f2(1.0f), e);
+      const float2 nq = __fmul2_rn(m2, rs);                // -sqrt(1 - alpha^2)
+      const float2 nix = __ffma2_rn(nhx, tanh2(hi), nhx);  // -i x
+      AL[s] = al;
+      NQ[s] = nq;
+      CP[s] = __ffma2_rn(__fmul2_rn(al, rs), nix, hc);
+      hc = __ffma2_rn(al, hc, __fmul2_rn(nq, nix));  // alpha h + sqrt(1 - alpha^2) i x
+    }
+  }
+#pragma unroll
+  for (int s = RB - 1; s >= 0; --s) {
+    if (FULL || s < srows) {
+      const float2 dh = bf2_unpack(*reinterpret_cast<const uint32_t*>(s_dh + s * ROWB));
+      const float2 nhx = bf2_scaled(lds_again(s_x + s * ROWB), kBf2NegHalf);
+      const float2 thr = tanh2(bf2_scaled(lds_again(s_r + s * ROWB), kBf2Half));
+      const float2 thi = tanh2(bf2_scaled(lds_again(s_i + s * ROWB), kBf2Half));
+      const float2 g = __fadd2_rn(dh, w);
+      w = __fmul2_rn(AL[s], g);
+      const float2 gnq = __fmul2_rn(g, NQ[s]);                    // -g sqrt(1 - alpha^2)
+      const float2 ni = __ffma2_rn(f2(-0.5f), thi, f2(-0.5f));    // -i
+      const float2 omi = __ffma2_rn(f2(-0.5f), thi, f2(0.5f));    // 1 - i
+      const float2 nix = __ffma2_rn(nhx, thi, nhx);               // -i x
+      const float2 ox = __fmul2_rn(gnq, ni);                      // g sqrt(1 - alpha^2) i
+      const float2 oi = __fmul2_rn(__fmul2_rn(gnq, nix), omi);    // g u (1 - i)
+      const float2 dl = __fmul2_rn(w, CP[s]);
+      const float2 orho = __fmul2_rn(dl, __ffma2_rn(nkq, __fmul2_rn(thr, thr), kq));
+      dlr = __ffma2_rn(dl, __ffma2_rn(f2(0.5f), thr, f2(0.5f)), dlr);  // += d l r
+      *reinterpret_cast<uint32_t*>(s_dh + s * ROWB) = bf2_pack(ox);
+      *reinterpret_cast<uint32_t*>(s_r + s * ROWB) = bf2_pack(orho);
+      *reinterpret_cast<uint32_t*>(s_i + s * ROWB) = bf2_pack(oi);
+    }
+  }
+}
+
 // MODE as seq_fwd_kernel's. kSeqSeg: block (segment s, chain) starts from the
 // adjoint carry that the maps (A, W) of the segments after s carry dh_last to,
 // and only segment 0 writes dh0.
@@ -522,6 +683,7 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
   constexpr uint32_t BOX = seq_box_bytes<T, VEC, R>();
   constexpr int NSUB = R / RB;
   static_assert(R % RB == 0, "sub-blocks must tile a stage");
+  constexpr bool kPacked = G::kHalfInputs && VEC == 2 && !GATED;  // as seq_fwd_kernel
   const Plan& p = a.p;
   extern __shared__ unsigned char seq_smem[];
   SeqRing<NB, BOX> ring{align128(seq_smem), nullptr, a.stages};
@@ -637,7 +799,25 @@ __global__ void __launch_bounds__(32, sizeof(T) == 4 ? 8 : 16) seq_bwd_kernel(co
           for (int v = 0; v < VEC; ++v) sq[u][v] = sq[u + 1][v];
         }
         if (m - QD >= 0) load_start(m - QD, sq[QD - 1]);  // in flight for QD sub-blocks
-        if (srows == RB) {
+        if constexpr (kPacked) {
+          float2 hc2 = make_float2(hc[0], hc[1]), w2 = make_float2(w[0], w[1]);
+          float2 dlr2 = make_float2(dlr[0], dlr[1]);
+          const float2 kh2 = make_float2(kh[0], kh[1]);
+          const float2 kq = make_float2(0.25f * k[0], 0.25f * k[1]);
+          const float2 nkq = make_float2(-kq.x, -kq.y);
+          if (srows == RB) {
+            if (poly)
+              seq_bwd_sub_bf16x2<true, true, R, RB>(lb, row0, srows, kh2, kq, nkq, hc2, w2, dlr2);
+            else
+              seq_bwd_sub_bf16x2<false, true, R, RB>(lb, row0, srows, kh2, kq, nkq, hc2, w2, dlr2);
+          } else {
+            seq_bwd_sub_bf16x2<false, false, R, RB>(lb, row0, srows, kh2, kq, nkq, hc2, w2, dlr2);
+          }
+          w[0] = w2.x;
+          w[1] = w2.y;
+          dlr[0] = dlr2.x;
+          dlr[1] = dlr2.y;
+        } else if (srows == RB) {
           if (poly)
             seq_bwd_sub<IO, G, true, true, R, RB, GATED>(lb, row0, srows, k, kh, hc, w, dlr);
           else
