@@ -99,7 +99,7 @@ typedef struct {
  *           bytes per element);
  *   segmented: the serial kernels' kept states, 8 bytes per channel per
  *           segment (of 128 steps or more) and the chained forward's records
- *           (12 bytes per channel per 64 steps), laid over the tiled forward
+ *           (12 bytes per channel per 128 steps), laid over the tiled forward
  *           records, plus the tiled backward records (for the _varlen forms),
  *           under 0.95 bytes per element;
  * plus the float64 partial sums of dlambda and a small header (about 72 bytes

@@ -15,7 +15,11 @@
 //      tile n evaluates the gates of Sec. 3.2 for the slice from the stage
 //      (which is then released), folds it serially from a zero state (hl_t,
 //      and am_t = the product of the alphas so far minus one, so that h_t =
-//      hl_t + (1 + am_t) h_start) and publishes the slice's map (A - 1, U).
+//      hl_t + (1 + am_t) h_start), publishes the slice's map (A - 1, U) and
+//      parks the per-step hl_t, am_t in the block's tensor memory (TMEM: the
+//      warp's 32 lanes x 2 kChainSlice VEC columns of a slot, written 16
+//      columns at a time as the fold advances), off the register file until
+//      pass C needs them.
 //      Then pass C of tile n - kChainLag, whose entering states the scanners
 //      have found meanwhile: h_t = hl_t + (1 + am_t) h_start is written to global
 //      memory from registers (coalesced 128-byte rows), with the kept states
@@ -44,8 +48,8 @@
 
 namespace blr {
 
-constexpr int kChainStages = 7;             // ring stages per block
-constexpr int kChainLag = 5;                // pass C runs this many tiles behind pass A
+constexpr int kChainStages = 4;             // ring stages per block
+constexpr int kChainLag = 3;                // pass C runs this many tiles behind pass A
 constexpr int kChainSlots = kChainLag + 1;  // slice-map, starting-state and TMEM slots
 constexpr uint32_t kChainTmemCols = 512;    // TMEM columns the block allocates (all of them)
 constexpr int kChainScanners = 3;
@@ -104,20 +108,24 @@ __device__ __forceinline__ float2 map_apply2(float2 m, float2 h, float2 U) {
 }
 __device__ __forceinline__ float m_compose(float m1, float m2) { return fmaf(m1, m2, m1 + m2); }
 
-// Pass A for one lane: the gates of the TS rows of its warp's slice (as the
-// serial forward evaluates them), then the slice folded from a zero state.
-// On return hl[s] is the state after row s from a zero start and am[s] the
-// product of the alphas of rows 0 .. s minus one.
-template <class IO, class G, bool POLY, int TS>
-__device__ __forceinline__ void chain_fold(const unsigned char* lb, const float (&k)[IO::VEC],
-                                           const float (&kh)[IO::VEC], float (&hl)[TS][IO::VEC],
-                                           float (&am)[TS][IO::VEC]) {
+// Pass A for one lane, QS rows of its warp's slice at a time (the rows whose
+// states fill 16 TMEM columns): the gates of the rows (as the serial forward
+// evaluates them), then the fold continued from (H, M), the state and the
+// product of alphas minus one after the slice's earlier rows (zero at its
+// start). The per-row states go to park in TMEM column order: for row r and
+// channel v, park[2 (r VEC + v)] = H_r and park[2 (r VEC + v) + 1] = M_r.
+template <class IO, class G, bool POLY, int QS>
+__device__ __forceinline__ void chain_fold_part(const unsigned char* lb, const float (&k)[IO::VEC],
+                                                const float (&kh)[IO::VEC], float (&H)[IO::VEC],
+                                                float (&M)[IO::VEC], float (&park)[16]) {
   using Raw = typename IO::Raw;
   constexpr int V = IO::VEC;
+  static_assert(2 * QS * V == 16, "a part fills 16 columns");
   constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
   constexpr uint32_t BOX = kChainTile * ROWB;
+  float hl[QS][V], am[QS][V];
 #pragma unroll
-  for (int s = 0; s < TS; ++s) {
+  for (int s = 0; s < QS; ++s) {
     float xv[V], rv[V], iv[V];
     if constexpr (G::kHalfInputs) {
       IO::unpack_half(*reinterpret_cast<const Raw*>(lb + s * ROWB), xv);
@@ -143,61 +151,49 @@ __device__ __forceinline__ void chain_fold(const unsigned char* lb, const float 
   }
 #pragma unroll
   for (int v = 0; v < V; ++v) {
-    float H = 0.0f, m = 0.0f;
 #pragma unroll
-    for (int s = 0; s < TS; ++s) {
+    for (int s = 0; s < QS; ++s) {
       const float e = am[s][v], alpha = 1.0f + e;
-      H = fmaf(alpha, H, hl[s][v]);
-      m = fmaf(alpha, m, e);  // alpha (1 + m) - 1
-      hl[s][v] = H;
-      am[s][v] = m;
+      H[v] = fmaf(alpha, H[v], hl[s][v]);
+      M[v] = fmaf(alpha, M[v], e);  // alpha (1 + M) - 1
+      park[2 * (s * V + v)] = H[v];
+      park[2 * (s * V + v) + 1] = M[v];
     }
   }
 }
 
-// Pass A for a bfloat16 lane (two channels, carried as one float2 so that the
-// multiply-adds run as packed pairs): the same arithmetic, in the same order,
-// as chain_fold with GatesFast.
-template <bool POLY, int TS>
-__device__ __forceinline__ void chain_fold_bf16x2(const unsigned char* lb, float2 kh,
-                                                  float2 (&hl)[TS], float2 (&am)[TS]) {
-  using IO = Io<__nv_bfloat16, 2>;
+// The same for a bfloat16 lane (two channels, carried as one float2 so that
+// the multiply-adds run as packed pairs): the same arithmetic, in the same
+// order, as chain_fold_part with GatesFast, on 4 rows.
+template <bool POLY>
+__device__ __forceinline__ void chain_fold_part_bf16x2(const unsigned char* lb, float2 kh, float2& H,
+                                                       float2& M, float (&park)[16]) {
+  constexpr int QS = 4;
   constexpr uint32_t ROWB = 128;
   constexpr uint32_t BOX = kChainTile * ROWB;
-  const float2 one = make_float2(1.0f, 1.0f), two = make_float2(2.0f, 2.0f);
+  float2 hl[QS], am[QS];
 #pragma unroll
-  for (int s = 0; s < TS; ++s) {
-    float xv[2], rv[2], iv[2];
-    IO::unpack_half(*reinterpret_cast<const uint32_t*>(lb + s * ROWB), xv);
-    IO::unpack_half(*reinterpret_cast<const uint32_t*>(lb + BOX + s * ROWB), rv);
-    IO::unpack_half(*reinterpret_cast<const uint32_t*>(lb + 2 * BOX + s * ROWB), iv);
+  for (int s = 0; s < QS; ++s) {
+    const float2 hx = bf2_scaled(*reinterpret_cast<const uint32_t*>(lb + s * ROWB), kBf2Half);
+    const float2 hr = bf2_scaled(*reinterpret_cast<const uint32_t*>(lb + BOX + s * ROWB), kBf2Half);
+    const float2 hi = bf2_scaled(*reinterpret_cast<const uint32_t*>(lb + 2 * BOX + s * ROWB), kBf2Half);
     // l = kh tanh(rho/2) + kh, e = e^l - 1
-    const float2 l = __ffma2_rn(kh, make_float2(tanh_approx(rv[0]), tanh_approx(rv[1])), kh);
-    float2 e;
-    if (POLY) {  // the degree-4 series of expm1_taylor<4>
-      float2 q = __ffma2_rn(make_float2(1.0f / 24, 1.0f / 24), l, make_float2(1.0f / 6, 1.0f / 6));
-      q = __ffma2_rn(q, l, make_float2(0.5f, 0.5f));
-      q = __ffma2_rn(q, l, one);
-      e = __fmul2_rn(q, l);
-    } else {
-      e = make_float2(expm1_neg<4, false>(l.x), expm1_neg<4, false>(l.y));
-    }
+    const float2 e = expm1_neg2<POLY>(__ffma2_rn(kh, tanh2(hr), kh));
     am[s] = e;
     // 1 - alpha^2 = -e (e + 2); u = sqrt(1 - alpha^2) i x with i x = (x/2) tanh(iota/2) + x/2
-    const float2 m = __fmul2_rn(e, __fadd2_rn(e, two));
-    const float2 gx = __ffma2_rn(make_float2(xv[0], xv[1]),
-                                 make_float2(tanh_approx(iv[0]), tanh_approx(iv[1])),
-                                 make_float2(xv[0], xv[1]));
-    hl[s] = __fmul2_rn(make_float2(sqrt_approx(-m.x), sqrt_approx(-m.y)), gx);
+    const float2 m2 = __fmul2_rn(e, __fadd2_rn(e, f2(2.0f)));
+    hl[s] = __fmul2_rn(make_float2(sqrt_approx(-m2.x), sqrt_approx(-m2.y)),
+                       __ffma2_rn(hx, tanh2(hi), hx));
   }
-  float2 H = make_float2(0.0f, 0.0f), m = make_float2(0.0f, 0.0f);
 #pragma unroll
-  for (int s = 0; s < TS; ++s) {
-    const float2 alpha = __fadd2_rn(one, am[s]);
+  for (int s = 0; s < QS; ++s) {
+    const float2 alpha = __fadd2_rn(f2(1.0f), am[s]);
     H = __ffma2_rn(alpha, H, hl[s]);
-    m = __ffma2_rn(alpha, m, am[s]);  // alpha (1 + m) - 1
-    hl[s] = H;
-    am[s] = m;
+    M = __ffma2_rn(alpha, M, am[s]);  // alpha (1 + M) - 1
+    park[4 * s] = H.x;
+    park[4 * s + 1] = M.x;
+    park[4 * s + 2] = H.y;
+    park[4 * s + 3] = M.y;
   }
 }
 
@@ -270,9 +266,11 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
   constexpr int LAG = kChainLag;
   constexpr uint32_t ROWB = CHW * sizeof(T);
   constexpr uint32_t BOX = chain_box_bytes<T, VEC>();
-  static_assert(2 * TS * VEC <= 16, "a lane's states of one tile fill at most 16 TMEM columns");
+  // A lane's states of one slice fill NP parts of 16 TMEM columns (QS rows each).
+  constexpr int QS = 16 / (2 * VEC), NP = TS / QS;
+  static_assert(QS * 2 * VEC == 16 && NP * QS == TS && NP <= 2, "slices of whole 16-column parts");
   static_assert(RB % TS == 0, "a slice holds at most one kept state, on its last row");
-  static_assert(NW % 4 == 0 && (NW / 4) * 16 * MS <= kChainTmemCols, "TMEM slots");
+  static_assert(NW % 4 == 0 && (NW / 4) * 16 * NP * MS <= kChainTmemCols, "TMEM slots");
   const Plan& p = a.p;
   extern __shared__ unsigned char chain_smem[];
   unsigned char* base = align128(chain_smem);
@@ -434,8 +432,9 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
     // C first, so that A's park store has a whole iteration to complete before
     // the next A waits for it.
     tmem_fence_after_sync();
-    const uint32_t tq = *tslot + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(warp >> 2) * 16;
-    constexpr uint32_t kSlotCols = (NW / 4) * 16;
+    constexpr uint32_t kWarpCols = 16 * NP;
+    constexpr uint32_t kSlotCols = (NW / 4) * kWarpCols;
+    const uint32_t tq = *tslot + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(warp >> 2) * kWarpCols;
     constexpr bool BF16X2 = G::kHalfInputs && VEC == 2;
     T* h = static_cast<T*>(a.h);
     float* kept = reinterpret_cast<float*>(a.ws + p.off_skept);
@@ -447,31 +446,35 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         // its parked states first (ready since its pass A), then its starting state
         const uint32_t q = n - LAG;
         const uint32_t m = q % MS;
-        uint32_t pr[16];
+        uint32_t pr[NP][16];
         __syncwarp();  // tcgen05 accesses are warp-collective
-        tmem_ld16_start(tq + m * kSlotCols, pr);
+#pragma unroll
+        for (int part = 0; part < NP; ++part) tmem_ld16_start(tq + m * kSlotCols + part * 16, pr[part]);
         mbar_wait(&carry_ready[m], (q / MS) & 1u, err);
         const int4 c = meta[m];
         float hs[VEC];
 #pragma unroll
         for (int v = 0; v < VEC; ++v) hs[v] = maps[(m * NW + warp) * CHW + lane * VEC + v].x;
         __syncwarp();
-        tmem_ld_wait(pr);
-        float park[16];
 #pragma unroll
-        for (int i2 = 0; i2 < 16; ++i2) park[i2] = __uint_as_float(pr[i2]);
+        for (int part = 0; part < NP; ++part) tmem_ld_wait(pr[part]);
         float out[TS][VEC];
 #pragma unroll
         for (int r = 0; r < TS; ++r) {
+          const uint32_t* pk = pr[r / QS];
+          const int r0 = r % QS;
           if constexpr (BF16X2) {
-            const float2 o = map_apply2(make_float2(park[4 * r + 1], park[4 * r + 3]),
-                                        make_float2(hs[0], hs[1]), make_float2(park[4 * r], park[4 * r + 2]));
+            const float2 o = map_apply2(
+                make_float2(__uint_as_float(pk[4 * r0 + 1]), __uint_as_float(pk[4 * r0 + 3])),
+                make_float2(hs[0], hs[1]),
+                make_float2(__uint_as_float(pk[4 * r0]), __uint_as_float(pk[4 * r0 + 2])));
             out[r][0] = o.x;
             out[r][1] = o.y;
           } else {
 #pragma unroll
             for (int v = 0; v < VEC; ++v)
-              out[r][v] = map_apply(park[2 * (r * VEC + v) + 1], hs[v], park[2 * (r * VEC + v)]);
+              out[r][v] = map_apply(__uint_as_float(pk[2 * (r0 * VEC + v) + 1]), hs[v],
+                                    __uint_as_float(pk[2 * (r0 * VEC + v)]));
           }
         }
         const uint32_t d0 = (uint32_t)c.z * CHW + lane * VEC;  // D < 2^24
@@ -481,10 +484,18 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
           const int64_t row0 = (int64_t)c.y * p.D + d0;  // (batch row, channel) offset of a state
           if (h != nullptr) {
             T* ph = h + ((int64_t)c.y * p.L + t0) * p.D + d0;
+            if (rows == TS) {
 #pragma unroll
-            for (int r = 0; r < TS; ++r) {
-              if (r < rows) IO::store(ph, out[r]);
-              ph += p.D;
+              for (int r = 0; r < TS; ++r) {
+                IO::store(ph, out[r]);
+                ph += p.D;
+              }
+            } else {
+#pragma unroll
+              for (int r = 0; r < TS; ++r) {
+                if (r < rows) IO::store(ph, out[r]);
+                ph += p.D;
+              }
             }
           }
           // the slice's last row is a kept state when it ends a block of RB steps
@@ -510,62 +521,57 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         }
       }
       if (n < nmy) {
-        // ---- A: tile n's gates and slice fold; the stage is free again afterwards
+        // ---- A: tile n's gates and slice fold, parked 16 columns at a time;
+        // the stage is free again afterwards
         const uint32_t s = n % S, m = n % MS;
-        tmem_wait_st();  // the previous tile's park store, before a later load of its slot
+        tmem_wait_st();  // the previous tile's park stores, before a later load of their slot
         mbar_wait(&full[s], (n / S) & 1u, err);
         const unsigned char* lb = base + s * (NB * BOX) + loff;
-        float park[16];
+        const bool poly = polys[s] != 0;
         float2 mapv[VEC];
         if constexpr (BF16X2) {
           const float2 r0 = rates[s * CHW + lane * 2], r1 = rates[s * CHW + lane * 2 + 1];
           const float2 kh = make_float2(r0.y, r1.y);
-          float2 hl[TS], am[TS];
-          if (polys[s])
-            chain_fold_bf16x2<true, TS>(lb, kh, hl, am);
-          else
-            chain_fold_bf16x2<false, TS>(lb, kh, hl, am);
+          float2 H = make_float2(0.0f, 0.0f), M = make_float2(0.0f, 0.0f);
 #pragma unroll
-          for (int r = 0; r < TS; ++r) {
-            park[4 * r] = hl[r].x;
-            park[4 * r + 1] = am[r].x;
-            park[4 * r + 2] = hl[r].y;
-            park[4 * r + 3] = am[r].y;
+          for (int part = 0; part < NP; ++part) {
+            float park[16];
+            if (poly)
+              chain_fold_part_bf16x2<true>(lb + part * QS * ROWB, kh, H, M, park);
+            else
+              chain_fold_part_bf16x2<false>(lb + part * QS * ROWB, kh, H, M, park);
+            __syncwarp();
+            tmem_st16(tq + m * kSlotCols + part * 16, park);
           }
-          mapv[0] = make_float2(am[TS - 1].x, hl[TS - 1].x);
-          mapv[1] = make_float2(am[TS - 1].y, hl[TS - 1].y);
+          mapv[0] = make_float2(M.x, H.x);
+          mapv[1] = make_float2(M.y, H.y);
         } else {
-          float k[VEC], kh[VEC];
+          float k[VEC], kh[VEC], H[VEC], M[VEC];
 #pragma unroll
           for (int v = 0; v < VEC; ++v) {
             const float2 r = rates[s * CHW + lane * VEC + v];
             k[v] = r.x;
             kh[v] = r.y;
-          }
-          float hl[TS][VEC], am[TS][VEC];
-          if (polys[s])
-            chain_fold<IO, G, true, TS>(lb, k, kh, hl, am);
-          else
-            chain_fold<IO, G, false, TS>(lb, k, kh, hl, am);
-#pragma unroll
-          for (int i2 = 0; i2 < 16; ++i2) park[i2] = 0.0f;
-#pragma unroll
-          for (int r = 0; r < TS; ++r) {
-#pragma unroll
-            for (int v = 0; v < VEC; ++v) {
-              park[2 * (r * VEC + v)] = hl[r][v];
-              park[2 * (r * VEC + v) + 1] = am[r][v];
-            }
+            H[v] = 0.0f;
+            M[v] = 0.0f;
           }
 #pragma unroll
-          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(am[TS - 1][v], hl[TS - 1][v]);
+          for (int part = 0; part < NP; ++part) {
+            float park[16];
+            if (poly)
+              chain_fold_part<IO, G, true, QS>(lb + part * QS * ROWB, k, kh, H, M, park);
+            else
+              chain_fold_part<IO, G, false, QS>(lb + part * QS * ROWB, k, kh, H, M, park);
+            __syncwarp();
+            tmem_st16(tq + m * kSlotCols + part * 16, park);
+          }
+#pragma unroll
+          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(M[v], H[v]);
         }
         mbar_arrive(&empty[s]);  // the stage is read: the producer may refill it
 #pragma unroll
         for (int v = 0; v < VEC; ++v) maps[(m * NW + warp) * CHW + lane * VEC + v] = mapv[v];
         mbar_arrive(&maps_ready[m]);
-        __syncwarp();
-        tmem_st16(tq + m * kSlotCols, park);
       }
     }
     tmem_wait_st();

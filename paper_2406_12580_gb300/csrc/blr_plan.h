@@ -86,7 +86,7 @@ constexpr int64_t kSeqTallRowsMinL = 1024;
 // tile (a warp slice of kChainSlice steps), chained along time by a decoupled
 // look-back over per-(tile, channel) records.
 constexpr int kChainWarps = 16;
-constexpr int kChainSlice = 4;
+constexpr int kChainSlice = 8;
 constexpr int kChainTile = kChainWarps * kChainSlice;
 
 constexpr int64_t kSegMinL = 2048;

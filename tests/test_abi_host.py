@@ -194,7 +194,7 @@ def test_workspace_bytes(lib):
         assert wb(B, L, Dd, io) < 0.5 * n + 64 * Dd + 4096, (B, L, Dd)
     # segmented problems keep the serial kernels' states, 8 bytes per channel
     # per segment of 128 steps or more, the chained forward's records (12 bytes
-    # per channel per 64 steps) and the tiled backward records
+    # per channel per 128 steps) and the tiled backward records
     for B, L, Dd, io in ((8, 32768, 512, 1), (64, 2048, 64, 1), (3, 100000, 64, 1), (1, 65536, 8, 1)):
         n = B * L * Dd
         assert wb(B, L, Dd, io) < 0.95 * n + 24 * B * Dd + 64 * Dd + 4096, (B, L, Dd)
