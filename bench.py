@@ -32,6 +32,7 @@ import dataclasses
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -121,12 +122,22 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def code_text(src: str) -> str:
+    """A CUDA/C++ source without its comments and blank lines, each line
+    stripped: what the compiler sees, so that a comment edit leaves it alone."""
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    lines = (re.sub(r"//.*", "", ln).strip() for ln in src.splitlines())
+    return "\n".join(ln for ln in lines if ln)
+
+
 def kernel_sources_sha() -> str:
+    """Hash of the library's code (comments excluded), which the committed ncu
+    traffic figures are tied to."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2406_12580_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode() + b"\0" + f.read())
+        with open(os.path.join(csrc, name), encoding="utf-8") as f:
+            h.update(name.encode() + b"\0" + code_text(f.read()).encode())
     return h.hexdigest()[:16]
 
 
@@ -614,7 +625,8 @@ def e2e_pipelined(inp, reps, world, dev, nsets=3):
 
 def other_workloads(flush, peak, peak_kind, dev, headline):
     """The other workloads (parity-test shapes beside the headline), each with
-    per-call rooflines; L2 flushed before every call; and the recurrent step."""
+    per-call rooflines; L2 flushed before every call; the recurrent step; and
+    one training step of the gated recurrent layer (tokens/s)."""
     import torch
     from paper_2406_12580_gb300 import inputs as I
     from paper_2406_12580_gb300.device import ScanBuffers, StepBuffers
@@ -641,6 +653,9 @@ def other_workloads(flush, peak, peak_kind, dev, headline):
         del sbuf
     g = step_graph(flush, peak, dev)
     out["step_f32_graph8"] = {"us": round(g["ms_per_step"] * 1e3, 2), "frac": round(g["frac"], 3)}
+    t = layer_workload(flush, dev, serial=False)
+    out["layer_train_step"] = {"ms": round(t["ms_fused_kernels"], 3),
+                               "tokens_per_s": round(t["tokens_per_s"])}
     return out
 
 
@@ -759,17 +774,23 @@ def padding_table(flush, dev, B=256, D=64, reps=20):
             "rows": rows}
 
 
-def layer_workload(flush, dev, B=256, L=200, D=64, E=2, reps=10):
-    """One training step (forward and backward) of the gated recurrent layer
-    of Alg. 1 (layer.GatedRecurrentLayer: torch GEMMs and convolution, the scan
-    and merge on the library's kernels) against the same layer with the scan as
-    a step-by-step torch loop on the GPU (a serial scan)."""
+def layer_workload(flush, dev, B=256, L=200, D=64, E=2, reps=10, serial=True):
+    """One training step (forward, backward and an Adam update, lr 1e-3) of the
+    gated recurrent layer of Alg. 1 (layer.GatedRecurrentLayer: torch GEMMs and
+    convolution, the scan and merge on the library's kernels), and (serial)
+    the same step with the scan as a step-by-step torch loop on the GPU."""
     import torch
     from paper_2406_12580_gb300.layer import GatedRecurrentLayer
     torch.manual_seed(0)
     layer = GatedRecurrentLayer(D, expand=E, device=dev)
+    opt = torch.optim.Adam(layer.parameters(), lr=1e-3)
     h = torch.randn(B, L, D, device=dev, requires_grad=True)
     g = torch.randn(B, L, D, device=dev)
+
+    def train_step(fwd):
+        opt.zero_grad(set_to_none=False)
+        (fwd(h) * g).sum().backward()
+        opt.step()
 
     def serial_forward(x_in):
         hx, hz = layer.in_proj(x_in).split(layer.ed, dim=-1)
@@ -786,24 +807,27 @@ def layer_workload(flush, dev, B=256, L=200, D=64, E=2, reps=10):
         return layer.out_proj(torch.stack(hs, dim=1) * torch.nn.functional.silu(hz))
 
     res = {}
-    for name, fwd in (("fused_kernels", layer), ("serial_torch_scan", serial_forward)):
+    variants = (("fused_kernels", layer), ("serial_torch_scan", serial_forward))
+    for name, fwd in variants if serial else variants[:1]:
         n = reps if name == "fused_kernels" else max(2, reps // 5)
         for _ in range(2):
-            (fwd(h) * g).sum().backward()
+            train_step(fwd)
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in range(n)]
         for e0, e1 in ev:
             flush()
             e0.record()
-            (fwd(h) * g).sum().backward()
+            train_step(fwd)
             e1.record()
         torch.cuda.synchronize()
         res[name] = statistics.median(a.elapsed_time(b) for a, b in ev)
-    return {"workload": f"gated recurrent layer (Alg. 1) d_model={D} E={E} B={B} L={L} f32, "
-                        "forward + backward", "ms_fused_kernels": res["fused_kernels"],
-            "ms_serial_torch_scan": res["serial_torch_scan"],
-            "tokens_per_s": B * L / (res["fused_kernels"] * 1e-3),
-            "serial_over_fused": res["serial_torch_scan"] / res["fused_kernels"]}
+    out = {"workload": f"gated recurrent layer (Alg. 1) d_model={D} E={E} B={B} L={L} f32, "
+                       "forward + backward + Adam", "ms_fused_kernels": res["fused_kernels"],
+           "tokens_per_s": B * L / (res["fused_kernels"] * 1e-3)}
+    if serial:
+        out.update(ms_serial_torch_scan=res["serial_torch_scan"],
+                   serial_over_fused=res["serial_torch_scan"] / res["fused_kernels"])
+    return out
 
 
 def gated_workload(k, flush, peak, dev, reps=20):
