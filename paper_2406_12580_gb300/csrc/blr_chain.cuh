@@ -268,8 +268,8 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
   constexpr uint32_t BOX = chain_box_bytes<T, VEC>();
   // A lane's states of one slice fill NP parts of 16 TMEM columns (QS rows each).
   constexpr int QS = 16 / (2 * VEC), NP = TS / QS;
-  static_assert(QS * 2 * VEC == 16 && NP * QS == TS && NP <= 2, "slices of whole 16-column parts");
-  static_assert(RB % TS == 0, "a slice holds at most one kept state, on its last row");
+  static_assert(QS * 2 * VEC == 16 && NP * QS == TS && NP <= 4, "slices of whole 16-column parts");
+  static_assert(RB % TS == 0 || TS % RB == 0, "kept states fall on slice rows");
   static_assert(NW % 4 == 0 && (NW / 4) * 16 * NP * MS <= kChainTmemCols, "TMEM slots");
   const Plan& p = a.p;
   extern __shared__ unsigned char chain_smem[];
@@ -498,8 +498,18 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
               }
             }
           }
-          // the slice's last row is a kept state when it ends a block of RB steps
-          if (rows == TS && (t0 + TS) % RB == 0) {
+          // kept states: the rows that end a block of RB steps (a slice's last
+          // row, or every RB-th row of a slice that spans several blocks)
+          if constexpr (TS % RB == 0) {
+#pragma unroll
+            for (int r = RB - 1; r < TS; r += RB) {
+              const int64_t mk = (t0 + r + 1) / RB - 1;
+              if (r < rows && mk < p.n_carry) {
+#pragma unroll
+                for (int v = 0; v < VEC; ++v) kept[mk * BD + row0 + v] = out[r][v];
+              }
+            }
+          } else if (rows == TS && (t0 + TS) % RB == 0) {
             const int64_t mk = (t0 + TS) / RB - 1;
             if (mk < p.n_carry) {
 #pragma unroll
