@@ -144,15 +144,15 @@ def kernel_sources_sha() -> str:
 def scan_kernels(cfg):
     """(forward kernels, backward kernels, our kernels per forward call, per
     backward call) of the family the library runs on this shape
-    (blr_scan_family). The chained forward also clears its records with one
-    cudaMemsetAsync, which is not counted as a kernel of ours."""
+    (blr_scan_family). The chained kernels also clear their records with one
+    cudaMemsetAsync a call, which is not counted as a kernel of ours."""
     from paper_2406_12580_gb300 import (FAMILY_SEGMENTED, FAMILY_SERIAL, Desc,
                                         blr_scan_family)
     fam = blr_scan_family(Desc(cfg.B, cfg.L, cfg.D, 0 if cfg.io == "f32" else 1, cfg.c))
     if fam == FAMILY_SERIAL:
         return "seq_fwd_kernel", "seq_bwd_kernel", 1, 1
     if fam == FAMILY_SEGMENTED:
-        return "chain_fwd_kernel", "seg_reduce_kernel+seq_bwd_kernel", 1, 2
+        return "chain_fwd_kernel", "chain_bwd_kernel", 1, 1
     return "prep_kernel+scan_fwd_kernel", "prep_kernel+scan_bwd_kernel", 2, 2
 
 

@@ -13,6 +13,7 @@
 
 #include "blr.h"
 #include "blr_chain.cuh"
+#include "blr_chain_bwd.cuh"
 #include "blr_merge.cuh"
 #include "blr_seq.cuh"
 
@@ -468,6 +469,36 @@ blr_status scan_fwd_chain(const Plan& plan, const void* x, const void* gl, const
   return launch_chain_fwd<__nv_bfloat16, blr::MathFast, 2, 8>(plan, a, st);
 }
 
+// The chained single-pass backward (the problems the chained forward serves,
+// bfloat16): the records are emptied again (the forward's are no longer
+// needed), then one cooperative grid, one block per SM.
+blr_status scan_bwd_chain(const Plan& plan, const void* dh, const float* dh_last, const void* x,
+                          const void* gl, const float* lambda, const float* h0, void* dx, void* dgl,
+                          float* dlambda, float* dh0, unsigned char* w, cudaStream_t st) {
+  if (plan.io != BLR_BF16) return fail(BLR_ERR_UNSUPPORTED, "the chained backward takes bfloat16 I/O");
+  BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_cinc, 0xff, plan.off_cend - plan.off_cinc, st),
+                     "empty the chained backward's records"));
+  blr::ChainBwdArgs a;
+  BLR_TRY(seq_maps_x(&a.tm_dh, dh, plan, blr::kChainTile));
+  BLR_TRY(seq_maps_x(&a.tm_x, x, plan, blr::kChainTile));
+  BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, blr::kChainTile));
+  a.p = plan;
+  a.dh_last = dh_last;
+  a.lambda = lambda;
+  a.h0 = h0;
+  a.dx = dx;
+  a.dgl = dgl;
+  a.dlambda = dlambda;
+  a.dh0 = dh0;
+  a.ws = w;
+  using bf = __nv_bfloat16;
+  auto k = blr::chain_bwd_kernel<bf, blr::MathFast, 2, 8>;
+  const size_t smem = blr::ChainBwdSmem<bf, 2>::bytes;
+  unsigned grid = 1;
+  BLR_TRY(persistent_grid(k, blr::kCbThreads, smem, plan.n_tc * plan.n_chain, &grid));
+  return launch_cooperative(k, grid, blr::kCbThreads, smem, st, a, "launch chain_bwd_kernel");
+}
+
 // Clears [zero, zero + zero_bytes), fills [fill, fill + fill_bytes) with the
 // empty record pattern and writes k = -c softplus(Lambda).
 blr_status launch_prep(unsigned char* zero, size_t zero_bytes, unsigned char* fill,
@@ -710,9 +741,13 @@ blr_status scan_bwd_entry(const blr_desc* desc, const void* dh, const float* dh_
   if (plan.seq)  // the forward cleared the counters and partial sums
     return scan_bwd_seq(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
                         dh0, w, st, z, dz, lengths);
-  if (plan.nseg > 0 && lengths == nullptr)
+  if (plan.nseg > 0 && lengths == nullptr) {
+    if (z == nullptr)
+      return scan_bwd_chain(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
+                            dlambda, dh0, w, st);
     return scan_bwd_seg(plan, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits, dlambda,
                         dh0, w, st, z, dz);
+  }
   if (z == nullptr)
     return scan_bwd_tiled(plan, desc, dh, dh_last, x, gate_logits, lambda, h0, dx, dgate_logits,
                           dlambda, dh0, w, st, lengths);

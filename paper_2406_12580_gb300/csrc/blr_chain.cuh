@@ -199,10 +199,12 @@ __device__ __forceinline__ void chain_fold_part_bf16x2(const unsigned char* lb, 
 
 // ---------------------------------------------------------------- look-back
 //
-// One channel's walk. Predecessor j (a time block before the tile's) has its
-// records at inc[j * BD] and agg[j * BD]. kChainWindow predecessors, nearest
-// first, are read in one round trip; the walk folds aggregates until it meets
-// a published state. Time block 0 publishes only its state, so every walk ends.
+// One channel's walk over the tile's nprev predecessors, nearest first: the
+// q-th has its records at inc[q * step] and agg[q * step] (step = -BD when
+// the predecessors are the earlier time blocks, as in the forward; +BD when
+// they are the later ones, as in the backward). kChainWindow predecessors are
+// read in one round trip; the walk folds aggregates until it meets a published
+// state. The farthest predecessor publishes only its state, so every walk ends.
 
 struct ChainWindow {
   uint32_t in[kChainWindow];
@@ -210,24 +212,26 @@ struct ChainWindow {
 };
 
 __device__ __forceinline__ void chain_window_load(const unsigned long long* agg, const uint32_t* inc,
-                                                  int64_t BD, int64_t j, ChainWindow& w) {
+                                                  int64_t step, int64_t q0, int64_t nprev,
+                                                  ChainWindow& w) {
 #pragma unroll
   for (int q = 0; q < kChainWindow; ++q) {
     w.in[q] = kEmpty;
     w.ag[q] = ~0ull;
-    if (j - q >= 0) {
-      w.in[q] = ld_record(inc + (j - q) * BD);
-      w.ag[q] = ld_record(agg + (j - q) * BD);
+    if (q0 + q < nprev) {
+      w.in[q] = ld_record(inc + (q0 + q) * step);
+      w.ag[q] = ld_record(agg + (q0 + q) * step);
     }
   }
 }
 
-// The state entering the tile whose nearest predecessor is j, starting from
-// the window `w` already loaded for j. On an expired wait (recorded in *err)
-// it returns what it has.
+// The value entering the tile (its predecessors' state, or adjoint, carried
+// through them), starting from the window `w` already loaded for q0 = 0. On an
+// expired wait (recorded in *err) it returns what it has.
 __device__ __forceinline__ float chain_walk(const unsigned long long* agg, const uint32_t* inc,
-                                           int64_t BD, int64_t j, uint32_t* err, ChainWindow& w) {
+                                           int64_t step, int64_t nprev, uint32_t* err, ChainWindow& w) {
   float em = 0.0f, eu = 0.0f;  // the fold of the aggregates walked so far: h -> (1 + em) h + eu
+  int64_t q0 = 0;
   for (;;) {
     int adv = kChainWindow;
     bool open = true, wait = false;
@@ -245,11 +249,11 @@ __device__ __forceinline__ float chain_walk(const unsigned long long* agg, const
         }
       }
     }
-    if (j - adv < 0) return eu;  // no predecessor left (cannot happen: block 0 publishes its state)
-    if (wait && !wait_record(inc + (j - adv) * BD, agg + (j - adv) * BD, err, kWaitTimeoutNs))
+    if (q0 + adv >= nprev) return eu;  // no predecessor left (cannot happen: the farthest publishes its state)
+    if (wait && !wait_record(inc + (q0 + adv) * step, agg + (q0 + adv) * step, err, kWaitTimeoutNs))
       return eu;  // the wait expired (recorded): finish with what is known
-    j -= adv;
-    chain_window_load(agg, inc, BD, j, w);
+    q0 += adv;
+    chain_window_load(agg, inc, step, q0, nprev, w);
   }
 }
 
@@ -398,13 +402,13 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         } else {
 #pragma unroll
           for (int v = 0; v < VEC; ++v) st_record(&agg[rec + v], pack_agg(TM[v], TU[v]));
+          // predecessors: time blocks c.x - 1, c.x - 2, ..., 0
+          const int64_t near = rec - BD;
           ChainWindow win[VEC];
 #pragma unroll
-          for (int v = 0; v < VEC; ++v)
-            chain_window_load(agg + ch0 + v, inc + ch0 + v, BD, c.x - 1, win[v]);
+          for (int v = 0; v < VEC; ++v) chain_window_load(agg + near + v, inc + near + v, -BD, 0, c.x, win[v]);
 #pragma unroll
-          for (int v = 0; v < VEC; ++v)
-            hs[v] = chain_walk(agg + ch0 + v, inc + ch0 + v, BD, c.x - 1, err, win[v]);
+          for (int v = 0; v < VEC; ++v) hs[v] = chain_walk(agg + near + v, inc + near + v, -BD, c.x, err, win[v]);
         }
 #pragma unroll
         for (int v = 0; v < VEC; ++v) st_record(&inc[rec + v], __float_as_uint(map_apply(TM[v], hs[v], TU[v])));
