@@ -13,8 +13,9 @@
 // roles:
 //   producers (2 warps): one loads tile n's dh and rho into ring A; the other,
 //      a little before pass C needs it, tile n's x, rho and iota into ring C
-//      (rho is by then in L2). The first also writes the tiles' decay
-//      constants into a small ring of their own;
+//      (rho is by then in L2). The first also writes each tile's decay
+//      constants and coordinates into a small ring of their own, so that the
+//      compute warps divide no tile index;
 //   compute (kCbWarps warps, a slice of kCbSlice steps each, which starts at
 //      one of the forward's kept states): pass A of tile n evaluates the alphas
 //      of its slice and folds the reverse recurrence from a zero carry, last
@@ -49,7 +50,7 @@ constexpr int kCbThreads = (kCbWarps + kCbScanners + 2) * 32;
 constexpr uint32_t kCbTmemCols = 512;
 // Registers per thread, as kChainMaxRegs.
 constexpr int kCbMaxRegs = (16384 / (((kCbThreads / 32 + 3) / 4) * 32)) / 8 * 8;
-// Tiles' decay constants, a ring indexed by tile: the ring-A producer writes
+// Tiles' decay constants and coordinates, a ring indexed by tile: the ring-A producer writes
 // tile i's once pass A of tile i - kCbStagesA has freed its stage, and pass C
 // of tile i - kCbStagesA - kCbLag + 1 may still be to run.
 constexpr int kCbRates = 8;
@@ -82,7 +83,8 @@ struct ChainBwdSmem {
   static constexpr size_t ringC = ringA + (size_t)kCbStagesA * 2 * BOX;      // [SC][x, rho, iota]
   static constexpr size_t rates = ringC + (size_t)kCbStagesC * 3 * BOX;     // float2 [kCbRates][CHW]
   static constexpr size_t poly = up(rates + (size_t)kCbRates * CHW * sizeof(float2));  // int [kCbRates]
-  static constexpr size_t maps = up(poly + (size_t)kCbRates * sizeof(int));  // float2 [MS][W][CHW]
+  static constexpr size_t tmeta = up(poly + (size_t)kCbRates * sizeof(int));  // int4 [kCbRates]
+  static constexpr size_t maps = up(tmeta + (size_t)kCbRates * sizeof(int4));  // float2 [MS][W][CHW]
   static constexpr size_t meta = up(maps + (size_t)kCbSlots * kCbWarps * CHW * sizeof(float2));  // int4 [MS]
   static constexpr size_t tmem = up(meta + (size_t)kCbSlots * sizeof(int4));
   static constexpr size_t bars = up(tmem + sizeof(uint32_t));
@@ -204,6 +206,7 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
   unsigned char* base = align128(chain_smem);
   float2* rates = reinterpret_cast<float2*>(base + SM::rates);  // [kCbRates][CHW]: (k, k/2)
   int* polys = reinterpret_cast<int*>(base + SM::poly);
+  int4* tmeta = reinterpret_cast<int4*>(base + SM::tmeta);  // [kCbRates]: tile coordinates
   float2* maps = reinterpret_cast<float2*>(base + SM::maps);
   int4* meta = reinterpret_cast<int4*>(base + SM::meta);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(base + SM::tmem);
@@ -294,10 +297,13 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
       if (i >= SA) mbar_wait(&emptyA[s], (uint32_t)(i / SA - 1) & 1u, err);
 #pragma unroll
       for (int v = 0; v < VEC; ++v) rates[rr * CHW + lane * VEC + v] = make_float2(k[v], kh[v]);
-      if (lane == 0) polys[rr] = poly;
+      const int4 c = coord(i);
+      if (lane == 0) {
+        polys[rr] = poly;
+        tmeta[rr] = c;
+      }
       __syncwarp();
       if (lane == 0) {  // the arrival releases the constants with the stage
-        const int4 c = coord(i);
         unsigned char* dst = base + SM::ringA + (size_t)s * 2 * BOX;
         const int t = c.x * kChainTile, cd = c.z * CHW, cb = c.y;
         mbar_arrive_expect_tx(&fullA[s], 2 * BOX);
@@ -406,7 +412,7 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
         // ---- C: tile n - LAG, forward in time from the forward's kept state
         const uint32_t q = n - LAG;
         const uint32_t m = q % MS, sc = q % SC;
-        const int4 c = coord(q);
+        const int4 c = tmeta[q % kCbRates];
         const int64_t d0 = (int64_t)c.z * CHW + lane * VEC;
         const int64_t t0 = (int64_t)c.x * kChainTile + warp * TS;
         const int64_t row0 = (int64_t)c.y * p.D + d0;  // (batch row, channel) offset of a state
@@ -469,12 +475,12 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
         // 3-0, each part parked as soon as it is folded; the stage is free
         // afterwards
         const uint32_t s = n % SA, m = n % MS;
-        const int4 c = coord(n);
+        tmem_wait_st();  // the previous tile's park stores, before a later load of their slot
+        mbar_wait(&fullA[s], (n / SA) & 1u, err);
+        const int4 c = tmeta[n % kCbRates];
         const int64_t t0 = (int64_t)c.x * kChainTile + warp * TS;
         const int valid = t0 >= p.L ? 0 : (p.L - t0 < TS ? (int)(p.L - t0) : TS);
         const int valid1 = valid > QS ? valid - QS : 0, valid0 = valid < QS ? valid : QS;
-        tmem_wait_st();  // the previous tile's park stores, before a later load of their slot
-        mbar_wait(&fullA[s], (n / SA) & 1u, err);
         const unsigned char* lb = base + SM::ringA + s * (2 * BOX) + loff;
         const uint32_t rn = n % kCbRates;
         const float2 kh = make_float2(rates[rn * CHW + lane * VEC].y, rates[rn * CHW + lane * VEC + 1].y);
