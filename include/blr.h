@@ -116,11 +116,16 @@ BLR_API size_t blr_workspace_bytes(const blr_desc* desc);
  *                         through the whole sequence (one kernel per call).
  *   BLR_FAMILY_SEGMENTED  bfloat16 I/O, fewer chains, L >= 2048 and either
  *                         at least 8 Mi elements or L >= 16384, without
- *                         lengths: each chain is cut into time segments of
- *                         128 steps or more; a reduction kernel computes every
- *                         segment's affine map (the operator of Sec. 3.3),
- *                         then one warp walks each segment from the carry the
- *                         maps compose (two kernels per call).
+ *                         lengths. blr_scan_fwd and blr_scan_bwd run one
+ *                         chained kernel each: 128-step tiles folded by 16
+ *                         warps and chained along time by a decoupled
+ *                         look-back (the operator of Sec. 3.3), after one
+ *                         cudaMemsetAsync that empties the look-back records.
+ *                         The _gated forms cut each chain into time segments
+ *                         of 128 steps or more: a reduction kernel computes
+ *                         every segment's affine map, then one warp walks each
+ *                         segment from the carry the maps compose (two kernels
+ *                         per call).
  *   BLR_FAMILY_TILED      otherwise: 64-step tiles chained by a decoupled
  *                         look-back (a preparation kernel, then the scan).
  *   BLR_FAMILY_NONE       an invalid or empty problem (nothing is launched).

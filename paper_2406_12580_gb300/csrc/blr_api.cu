@@ -482,12 +482,12 @@ blr_status scan_bwd_chain(const Plan& plan, const void* dh, const float* dh_last
   BLR_TRY(seq_maps_x(&a.tm_dh, dh, plan, blr::kChainTile));
   BLR_TRY(seq_maps_x(&a.tm_x, x, plan, blr::kChainTile));
   BLR_TRY(seq_maps_gl(&a.tm_r, &a.tm_i, gl, plan, blr::kChainTile));
+  BLR_TRY(seq_maps_x(&a.tm_dx, dx, plan, blr::kChainTile));
+  BLR_TRY(seq_maps_gl(&a.tm_dr, &a.tm_di, dgl, plan, blr::kChainTile));
   a.p = plan;
   a.dh_last = dh_last;
   a.lambda = lambda;
   a.h0 = h0;
-  a.dx = dx;
-  a.dgl = dgl;
   a.dlambda = dlambda;
   a.dh0 = dh0;
   a.ws = w;

@@ -546,41 +546,41 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         if constexpr (BF16X2) {
           const float2 r0 = rates[s * CHW + lane * 2], r1 = rates[s * CHW + lane * 2 + 1];
           const float2 kh = make_float2(r0.y, r1.y);
-          float2 H = make_float2(0.0f, 0.0f), M = make_float2(0.0f, 0.0f);
+          float2 H = make_float2(0.0f, 0.0f), Am = make_float2(0.0f, 0.0f);
 #pragma unroll
           for (int part = 0; part < NP; ++part) {
             float park[16];
             if (poly)
-              chain_fold_part_bf16x2<true>(lb + part * QS * ROWB, kh, H, M, park);
+              chain_fold_part_bf16x2<true>(lb + part * QS * ROWB, kh, H, Am, park);
             else
-              chain_fold_part_bf16x2<false>(lb + part * QS * ROWB, kh, H, M, park);
+              chain_fold_part_bf16x2<false>(lb + part * QS * ROWB, kh, H, Am, park);
             __syncwarp();
             tmem_st16(tq + m * kSlotCols + part * 16, park);
           }
-          mapv[0] = make_float2(M.x, H.x);
-          mapv[1] = make_float2(M.y, H.y);
+          mapv[0] = make_float2(Am.x, H.x);
+          mapv[1] = make_float2(Am.y, H.y);
         } else {
-          float k[VEC], kh[VEC], H[VEC], M[VEC];
+          float k[VEC], kh[VEC], H[VEC], Am[VEC];
 #pragma unroll
           for (int v = 0; v < VEC; ++v) {
             const float2 r = rates[s * CHW + lane * VEC + v];
             k[v] = r.x;
             kh[v] = r.y;
             H[v] = 0.0f;
-            M[v] = 0.0f;
+            Am[v] = 0.0f;
           }
 #pragma unroll
           for (int part = 0; part < NP; ++part) {
             float park[16];
             if (poly)
-              chain_fold_part<IO, G, true, QS>(lb + part * QS * ROWB, k, kh, H, M, park);
+              chain_fold_part<IO, G, true, QS>(lb + part * QS * ROWB, k, kh, H, Am, park);
             else
-              chain_fold_part<IO, G, false, QS>(lb + part * QS * ROWB, k, kh, H, M, park);
+              chain_fold_part<IO, G, false, QS>(lb + part * QS * ROWB, k, kh, H, Am, park);
             __syncwarp();
             tmem_st16(tq + m * kSlotCols + part * 16, park);
           }
 #pragma unroll
-          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(M[v], H[v]);
+          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(Am[v], H[v]);
         }
         mbar_arrive(&empty[s]);  // the stage is read: the producer may refill it
 #pragma unroll

@@ -13,7 +13,8 @@
 // roles:
 //   producers (2 warps): one loads tile n's dh and rho into ring A; the other,
 //      a little before pass C needs it, tile n's x, rho and iota into ring C
-//      (rho is by then in L2). The first also writes each tile's decay
+//      (rho is by then in L2), and once pass C has written the tile's outputs
+//      over them, sends those out by TMA store before refilling the stage. The first also writes each tile's decay
 //      constants and coordinates into a small ring of their own, so that the
 //      compute warps divide no tile index;
 //   compute (kCbWarps warps, a slice of kCbSlice steps each, which starts at
@@ -26,7 +27,8 @@
 //      has found the adjoint entering its slice: starting from the forward's
 //      kept state it re-runs the slice forward in time, recomputing each
 //      step's gates once, h_{t-1}, g_t and every output (dx, d rho, d iota and
-//      the d Lambda terms) in one sweep, and writes them from registers;
+//      the d Lambda terms) in one sweep, writing the outputs over the step's
+//      consumed inputs in the ring C stage;
 //   scanners (kCbScanners warps, tiles in turn): compose the slice maps into
 //      the tile's, chain it to the tiles after it by the decoupled look-back of
 //      the forward, publish the adjoint leaving the tile, and hand every slice
@@ -62,12 +64,13 @@ struct ChainBwdArgs {
   CUtensorMap tm_x;
   CUtensorMap tm_r;
   CUtensorMap tm_i;
+  CUtensorMap tm_dx;  // the outputs, stored from ring C by TMA
+  CUtensorMap tm_dr;
+  CUtensorMap tm_di;
   Plan p;
   const float* dh_last;
   const float* lambda;
   const float* h0;
-  void* dx;   // (B, L, D) io dtype
-  void* dgl;  // (B, L, 2D) io dtype
   float* dlambda;
   float* dh0;
   unsigned char* ws;
@@ -132,15 +135,15 @@ __device__ __forceinline__ void chain_bwd_fold_part_bf16x2(const unsigned char* 
 // slice: rows 0 .. QS-1 at lb forward in time from h before them (hp, updated
 // to h after them), each step's gates evaluated once (as the serial kernels
 // evaluate them) for the state, g_t = gl_t + (1 + sm_t) w_in and the
-// gradients; rows from `rows` on lie past the sequence and are neither written
-// nor summed. pr holds (gl, sm) of row r at [4r, 4r + 4); kq = k/4 and
+// gradients, which overwrite the row's x, rho and iota in the stage (dx,
+// d rho, d iota: the TMA store clips rows past the sequence); rows from `rows`
+// on are not summed. pr holds (gl, sm) of row r at [4r, 4r + 4); kq = k/4 and
 // nkq = -k/4 per channel. Adds the d Lambda terms dl_t r_t to dlr; dh0, if not
 // NULL, receives alpha_0 g_0 of the part's first row (the sequence's first).
 template <bool POLY>
-__device__ __forceinline__ void chain_bwd_rows(const unsigned char* lb, const uint32_t (&pr)[16],
-                                               float2 win, float2 kq, float2 nkq, float2 kh, int rows,
-                                               float2& hp, __nv_bfloat16* dx, __nv_bfloat16* dg,
-                                               int64_t D, float* dh0, float2& dlr) {
+__device__ __forceinline__ void chain_bwd_rows(unsigned char* lb, const uint32_t (&pr)[16], float2 win,
+                                               float2 kq, float2 nkq, float2 kh, int rows, float2& hp,
+                                               float* dh0, float2& dlr) {
   constexpr int QS = 4;
   constexpr uint32_t ROWB = 128;
   constexpr uint32_t BOX = kChainTile * ROWB;
@@ -170,18 +173,16 @@ __device__ __forceinline__ void chain_bwd_rows(const unsigned char* lb, const ui
     const float2 dl = __fmul2_rn(w, __ffma2_rn(__fmul2_rn(alpha, rs), nix, hp));
     const float2 orho = __fmul2_rn(dl, __ffma2_rn(nkq, __fmul2_rn(thr, thr), kq));
     hp = __ffma2_rn(alpha, hp, __fmul2_rn(nq, nix));  // alpha h + sqrt(1 - alpha^2) i x
+    *reinterpret_cast<uint32_t*>(lb + r * ROWB) = bf2_pack(ox);
+    *reinterpret_cast<uint32_t*>(lb + BOX + r * ROWB) = bf2_pack(orho);
+    *reinterpret_cast<uint32_t*>(lb + 2 * BOX + r * ROWB) = bf2_pack(oi);
     if (r < rows) {
       dlr = __ffma2_rn(dl, __ffma2_rn(f2(0.5f), thr, f2(0.5f)), dlr);  // += d l r
-      __stcs(reinterpret_cast<unsigned int*>(dx), bf2_pack(ox));
-      __stcs(reinterpret_cast<unsigned int*>(dg), bf2_pack(orho));
-      __stcs(reinterpret_cast<unsigned int*>(dg + D), bf2_pack(oi));
       if (dh0 != nullptr && r == 0) {  // the sequence's first step: dh0 = alpha_0 g_0
         dh0[0] = w.x;
         dh0[1] = w.y;
       }
     }
-    dx += D;
-    dg += 2 * D;
   }
 }
 
@@ -213,8 +214,8 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
   uint64_t* fullA = reinterpret_cast<uint64_t*>(base + SM::bars);
   uint64_t* emptyA = fullA + SA;
   uint64_t* fullC = emptyA + SA;
-  uint64_t* emptyC = fullC + SC;
-  uint64_t* maps_ready = emptyC + SC;
+  uint64_t* writtenC = fullC + SC;  // a ring C stage holds its tile's outputs
+  uint64_t* maps_ready = writtenC + SC;
   uint64_t* carry_ready = maps_ready + MS;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -250,7 +251,7 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
     }
     for (int s = 0; s < SC; ++s) {
       mbar_init(&fullC[s], 1);
-      mbar_init(&emptyC[s], NW * 32);
+      mbar_init(&writtenC[s], NW * 32);
     }
     for (int m = 0; m < MS; ++m) {
       mbar_init(&maps_ready[m], NW * 32);
@@ -313,20 +314,35 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
     }
   } else if (warp == NW + kCbScanners + 1) {
     // ---------------------------------------------------------- producer C
-    // Tile q's x, rho and iota into ring C once pass C of tile q - SC has
-    // freed the stage.
+    // Step q: once pass C of tile q - SC has written its outputs over its
+    // stage, sends them out (dx, d rho, d iota: three TMA stores, clipped to
+    // the tensors) and, as soon as the stores have read the stage, loads tile
+    // q's x, rho and iota into it.
     if (lane == 0) {
-      for (int64_t q = 0; q < n_my; ++q) {
+      for (int64_t q = 0; q < n_my + SC; ++q) {
         const int s = (int)(q % SC);
-        if (q >= SC) mbar_wait(&emptyC[s], (uint32_t)(q / SC - 1) & 1u, err);
-        const int4 c = coord(q);
-        unsigned char* dst = base + SM::ringC + (size_t)s * 3 * BOX;
-        const int t = c.x * kChainTile, cd = c.z * CHW, cb = c.y;
-        mbar_arrive_expect_tx(&fullC[s], 3 * BOX);
-        tma_load_3d(dst, &a.tm_x, &fullC[s], cd, t, cb);
-        tma_load_3d(dst + BOX, &a.tm_r, &fullC[s], cd, t, cb);
-        tma_load_3d(dst + 2 * BOX, &a.tm_i, &fullC[s], cd, t, cb);
+        unsigned char* stg = base + SM::ringC + (size_t)s * 3 * BOX;
+        if (q >= SC) {
+          const int64_t j = q - SC;
+          mbar_wait(&writtenC[s], (uint32_t)(j / SC) & 1u, err);
+          const int4 c = coord(j);
+          const int t = c.x * kChainTile, cd = c.z * CHW, cb = c.y;
+          tma_store_3d(&a.tm_dx, stg, cd, t, cb);
+          tma_store_3d(&a.tm_dr, stg + BOX, cd, t, cb);
+          tma_store_3d(&a.tm_di, stg + 2 * BOX, cd, t, cb);
+          bulk_commit();
+          bulk_wait_read<0>();  // the stage is free once the stores have read it
+        }
+        if (q < n_my) {
+          const int4 c = coord(q);
+          const int t = c.x * kChainTile, cd = c.z * CHW, cb = c.y;
+          mbar_arrive_expect_tx(&fullC[s], 3 * BOX);
+          tma_load_3d(stg, &a.tm_x, &fullC[s], cd, t, cb);
+          tma_load_3d(stg + BOX, &a.tm_r, &fullC[s], cd, t, cb);
+          tma_load_3d(stg + 2 * BOX, &a.tm_i, &fullC[s], cd, t, cb);
+        }
       }
+      bulk_wait_all();  // every store complete before the block ends
     }
     __syncwarp();
   } else if (warp >= NW) {
@@ -401,8 +417,6 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
     constexpr uint32_t kSlotCols = (NW / 4) * kWarpCols;
     constexpr int QS = 4;
     const uint32_t tq = *tslot + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(warp >> 2) * kWarpCols;
-    T* dxp = static_cast<T*>(a.dx);
-    T* dglp = static_cast<T*>(a.dgl);
     const float* kept = reinterpret_cast<const float*>(a.ws + p.off_skept);
     double* acc = reinterpret_cast<double*>(a.ws + p.off_dlam);
     const uint32_t loff = warp * TS * ROWB + lane * VEC * sizeof(T);  // this lane's first row
@@ -439,29 +453,25 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
         const bool poly = polys[rq] != 0;
         __syncwarp();
         tmem_ld_wait(pr);
-        const unsigned char* lb = base + SM::ringC + sc * (3 * BOX) + loff;
+        unsigned char* lb = base + SM::ringC + sc * (3 * BOX) + loff;
         const int rows = !ch_ok || t0 >= p.L ? 0 : (p.L - t0 < TS ? (int)(p.L - t0) : TS);
         const int rows0 = rows < QS ? rows : QS, rows1 = rows - rows0;
-        const int64_t off = ((int64_t)c.y * p.L + t0) * p.D + d0;  // (b, t0, d0) in x-shaped tensors
-        T* dxs = dxp + off;
-        T* dgs = dglp + 2 * off - d0;  // (b, t0, d0) of the gate-logit gradients
         float* pd0 = (t0 == 0 && ch_ok) ? a.dh0 : nullptr;
         if (pd0 != nullptr) pd0 += row0;
         float2 dlr = make_float2(0.0f, 0.0f);
         if (poly)
-          chain_bwd_rows<true>(lb, pr, win, kq, nkq, kh, rows0, hp, dxs, dgs, p.D, pd0, dlr);
+          chain_bwd_rows<true>(lb, pr, win, kq, nkq, kh, rows0, hp, pd0, dlr);
         else
-          chain_bwd_rows<false>(lb, pr, win, kq, nkq, kh, rows0, hp, dxs, dgs, p.D, pd0, dlr);
+          chain_bwd_rows<false>(lb, pr, win, kq, nkq, kh, rows0, hp, pd0, dlr);
         __syncwarp();
         tmem_ld16_start(tq + m * kSlotCols + 16, pr);
         tmem_ld_wait(pr);
         if (poly)
-          chain_bwd_rows<true>(lb + QS * ROWB, pr, win, kq, nkq, kh, rows1, hp, dxs + QS * p.D,
-                               dgs + 2 * QS * p.D, p.D, nullptr, dlr);
+          chain_bwd_rows<true>(lb + QS * ROWB, pr, win, kq, nkq, kh, rows1, hp, nullptr, dlr);
         else
-          chain_bwd_rows<false>(lb + QS * ROWB, pr, win, kq, nkq, kh, rows1, hp, dxs + QS * p.D,
-                                dgs + 2 * QS * p.D, p.D, nullptr, dlr);
-        mbar_arrive(&emptyC[sc]);  // the stage is read: the producer may refill it
+          chain_bwd_rows<false>(lb + QS * ROWB, pr, win, kq, nkq, kh, rows1, hp, nullptr, dlr);
+        fence_proxy_async_smem();  // this thread's outputs in the stage, visible to the TMA stores
+        mbar_arrive(&writtenC[sc]);
         // d Lambda: this slice's terms into the float64 partial sums (reductions
         // without a result, striped over batch rows)
         if (rows > 0) {
