@@ -454,6 +454,7 @@ blr_status launch_chain_fwd(const Plan& plan, const blr::ChainFwdArgs& a, cudaSt
 blr_status scan_fwd_chain(const Plan& plan, const void* x, const void* gl, const float* lambda,
                           const float* h0, void* h, float* h_last, unsigned char* w,
                           cudaStream_t st) {
+  if (plan.io != BLR_BF16) return fail(BLR_ERR_UNSUPPORTED, "the chained forward takes bfloat16 I/O");
   BLR_TRY(cuda_check(cudaMemsetAsync(w + plan.off_cinc, 0xff, plan.off_cend - plan.off_cinc, st),
                      "empty the chained forward's records"));
   blr::ChainFwdArgs a;
@@ -465,7 +466,6 @@ blr_status scan_fwd_chain(const Plan& plan, const void* x, const void* gl, const
   a.h = h;
   a.h_last = h_last;
   a.ws = w;
-  if (plan.io == BLR_F32) return launch_chain_fwd<float, blr::MathPrecise, 1, 16>(plan, a, st);
   return launch_chain_fwd<__nv_bfloat16, blr::MathFast, 2, 8>(plan, a, st);
 }
 

@@ -108,63 +108,12 @@ __device__ __forceinline__ float2 map_apply2(float2 m, float2 h, float2 U) {
 }
 __device__ __forceinline__ float m_compose(float m1, float m2) { return fmaf(m1, m2, m1 + m2); }
 
-// Pass A for one lane, QS rows of its warp's slice at a time (the rows whose
-// states fill 16 TMEM columns): the gates of the rows (as the serial forward
-// evaluates them), then the fold continued from (H, M), the state and the
-// product of alphas minus one after the slice's earlier rows (zero at its
-// start). The per-row states go to park in TMEM column order: for row r and
-// channel v, park[2 (r VEC + v)] = H_r and park[2 (r VEC + v) + 1] = M_r.
-template <class IO, class G, bool POLY, int QS>
-__device__ __forceinline__ void chain_fold_part(const unsigned char* lb, const float (&k)[IO::VEC],
-                                                const float (&kh)[IO::VEC], float (&H)[IO::VEC],
-                                                float (&M)[IO::VEC], float (&park)[16]) {
-  using Raw = typename IO::Raw;
-  constexpr int V = IO::VEC;
-  static_assert(2 * QS * V == 16, "a part fills 16 columns");
-  constexpr uint32_t ROWB = 32 * V * sizeof(typename IO::T);
-  constexpr uint32_t BOX = kChainTile * ROWB;
-  float hl[QS][V], am[QS][V];
-#pragma unroll
-  for (int s = 0; s < QS; ++s) {
-    float xv[V], rv[V], iv[V];
-    if constexpr (G::kHalfInputs) {
-      IO::unpack_half(*reinterpret_cast<const Raw*>(lb + s * ROWB), xv);
-      IO::unpack_half(*reinterpret_cast<const Raw*>(lb + BOX + s * ROWB), rv);
-      IO::unpack_half(*reinterpret_cast<const Raw*>(lb + 2 * BOX + s * ROWB), iv);
-#pragma unroll
-      for (int v = 0; v < V; ++v) {
-        const float e = expm1_neg<G::kDeg, POLY>(G::decay_log_half(rv[v], kh[v]));
-        am[s][v] = e;
-        hl[s][v] = G::sqrt(-e * (e + 2.0f)) * G::gated_x_half(iv[v], xv[v]);
-      }
-    } else {
-      IO::unpack(*reinterpret_cast<const Raw*>(lb + s * ROWB), xv);
-      IO::unpack(*reinterpret_cast<const Raw*>(lb + BOX + s * ROWB), rv);
-      IO::unpack(*reinterpret_cast<const Raw*>(lb + 2 * BOX + s * ROWB), iv);
-#pragma unroll
-      for (int v = 0; v < V; ++v) {
-        const float e = expm1_neg<G::kDeg, POLY>(G::decay_log(rv[v], k[v], kh[v]));
-        am[s][v] = e;
-        hl[s][v] = G::sqrt(-e * (e + 2.0f)) * (G::sigmoid(iv[v]) * xv[v]);
-      }
-    }
-  }
-#pragma unroll
-  for (int v = 0; v < V; ++v) {
-#pragma unroll
-    for (int s = 0; s < QS; ++s) {
-      const float e = am[s][v], alpha = 1.0f + e;
-      H[v] = fmaf(alpha, H[v], hl[s][v]);
-      M[v] = fmaf(alpha, M[v], e);  // alpha (1 + M) - 1
-      park[2 * (s * V + v)] = H[v];
-      park[2 * (s * V + v) + 1] = M[v];
-    }
-  }
-}
-
-// The same for a bfloat16 lane (two channels, carried as one float2 so that
-// the multiply-adds run as packed pairs): the same arithmetic, in the same
-// order, as chain_fold_part with GatesFast, on 4 rows.
+// Pass A for a bfloat16 lane (two channels, carried as one float2 so that the
+// multiply-adds run as packed pairs), the 4 rows of its warp's slice whose
+// states fill 16 TMEM columns: the gates of the rows (as the serial forward
+// evaluates them, GatesFast), then the fold continued from (H, M), the state
+// and the product of alphas minus one after the slice's earlier rows (zero at
+// its start). Row r's states go to park[4r, 4r + 4) as (H.x, M.x, H.y, M.y).
 template <bool POLY>
 __device__ __forceinline__ void chain_fold_part_bf16x2(const unsigned char* lb, float2 kh, float2& H,
                                                        float2& M, float (&park)[16]) {
@@ -270,6 +219,7 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
   constexpr int LAG = kChainLag;
   constexpr uint32_t ROWB = CHW * sizeof(T);
   constexpr uint32_t BOX = chain_box_bytes<T, VEC>();
+  static_assert(VEC == 2 && G::kHalfInputs, "the chained kernels are the bfloat16 path");
   // A lane's states of one slice fill NP parts of 16 TMEM columns (QS rows each).
   constexpr int QS = 16 / (2 * VEC), NP = TS / QS;
   static_assert(QS * 2 * VEC == 16 && NP * QS == TS && NP <= 4, "slices of whole 16-column parts");
@@ -439,7 +389,6 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
     constexpr uint32_t kWarpCols = 16 * NP;
     constexpr uint32_t kSlotCols = (NW / 4) * kWarpCols;
     const uint32_t tq = *tslot + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)(warp >> 2) * kWarpCols;
-    constexpr bool BF16X2 = G::kHalfInputs && VEC == 2;
     T* h = static_cast<T*>(a.h);
     float* kept = reinterpret_cast<float*>(a.ws + p.off_skept);
     const uint32_t loff = warp * TS * ROWB + lane * VEC * sizeof(T);  // this lane's first row
@@ -467,19 +416,12 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         for (int r = 0; r < TS; ++r) {
           const uint32_t* pk = pr[r / QS];
           const int r0 = r % QS;
-          if constexpr (BF16X2) {
-            const float2 o = map_apply2(
-                make_float2(__uint_as_float(pk[4 * r0 + 1]), __uint_as_float(pk[4 * r0 + 3])),
-                make_float2(hs[0], hs[1]),
-                make_float2(__uint_as_float(pk[4 * r0]), __uint_as_float(pk[4 * r0 + 2])));
-            out[r][0] = o.x;
-            out[r][1] = o.y;
-          } else {
-#pragma unroll
-            for (int v = 0; v < VEC; ++v)
-              out[r][v] = map_apply(__uint_as_float(pk[2 * (r0 * VEC + v) + 1]), hs[v],
-                                    __uint_as_float(pk[2 * (r0 * VEC + v)]));
-          }
+          const float2 o = map_apply2(
+              make_float2(__uint_as_float(pk[4 * r0 + 1]), __uint_as_float(pk[4 * r0 + 3])),
+              make_float2(hs[0], hs[1]),
+              make_float2(__uint_as_float(pk[4 * r0]), __uint_as_float(pk[4 * r0 + 2])));
+          out[r][0] = o.x;
+          out[r][1] = o.y;
         }
         const uint32_t d0 = (uint32_t)c.z * CHW + lane * VEC;  // D < 2^24
         const uint32_t t0 = (uint32_t)c.x * kChainTile + warp * TS;  // L < 2^31
@@ -542,46 +484,20 @@ __global__ void __maxnreg__(kChainMaxRegs) chain_fwd_kernel(const __grid_constan
         mbar_wait(&full[s], (n / S) & 1u, err);
         const unsigned char* lb = base + s * (NB * BOX) + loff;
         const bool poly = polys[s] != 0;
-        float2 mapv[VEC];
-        if constexpr (BF16X2) {
-          const float2 r0 = rates[s * CHW + lane * 2], r1 = rates[s * CHW + lane * 2 + 1];
-          const float2 kh = make_float2(r0.y, r1.y);
-          float2 H = make_float2(0.0f, 0.0f), Am = make_float2(0.0f, 0.0f);
+        const float2 r0 = rates[s * CHW + lane * 2], r1 = rates[s * CHW + lane * 2 + 1];
+        const float2 kh = make_float2(r0.y, r1.y);
+        float2 H = make_float2(0.0f, 0.0f), Am = make_float2(0.0f, 0.0f);
 #pragma unroll
-          for (int part = 0; part < NP; ++part) {
-            float park[16];
-            if (poly)
-              chain_fold_part_bf16x2<true>(lb + part * QS * ROWB, kh, H, Am, park);
-            else
-              chain_fold_part_bf16x2<false>(lb + part * QS * ROWB, kh, H, Am, park);
-            __syncwarp();
-            tmem_st16(tq + m * kSlotCols + part * 16, park);
-          }
-          mapv[0] = make_float2(Am.x, H.x);
-          mapv[1] = make_float2(Am.y, H.y);
-        } else {
-          float k[VEC], kh[VEC], H[VEC], Am[VEC];
-#pragma unroll
-          for (int v = 0; v < VEC; ++v) {
-            const float2 r = rates[s * CHW + lane * VEC + v];
-            k[v] = r.x;
-            kh[v] = r.y;
-            H[v] = 0.0f;
-            Am[v] = 0.0f;
-          }
-#pragma unroll
-          for (int part = 0; part < NP; ++part) {
-            float park[16];
-            if (poly)
-              chain_fold_part<IO, G, true, QS>(lb + part * QS * ROWB, k, kh, H, Am, park);
-            else
-              chain_fold_part<IO, G, false, QS>(lb + part * QS * ROWB, k, kh, H, Am, park);
-            __syncwarp();
-            tmem_st16(tq + m * kSlotCols + part * 16, park);
-          }
-#pragma unroll
-          for (int v = 0; v < VEC; ++v) mapv[v] = make_float2(Am[v], H[v]);
+        for (int part = 0; part < NP; ++part) {
+          float park[16];
+          if (poly)
+            chain_fold_part_bf16x2<true>(lb + part * QS * ROWB, kh, H, Am, park);
+          else
+            chain_fold_part_bf16x2<false>(lb + part * QS * ROWB, kh, H, Am, park);
+          __syncwarp();
+          tmem_st16(tq + m * kSlotCols + part * 16, park);
         }
+        const float2 mapv[VEC] = {make_float2(Am.x, H.x), make_float2(Am.y, H.y)};
         mbar_arrive(&empty[s]);  // the stage is read: the producer may refill it
 #pragma unroll
         for (int v = 0; v < VEC; ++v) maps[(m * NW + warp) * CHW + lane * VEC + v] = mapv[v];
