@@ -45,7 +45,7 @@ constexpr int kCbWarps = 16;                   // compute warps
 constexpr int kCbSlice = 8;                    // steps a warp takes of a tile
 constexpr int kCbStagesA = 2;                  // ring A stages (dh, rho)
 constexpr int kCbStagesC = 2;                  // ring C stages (x, rho, iota)
-constexpr int kCbLag = 2;                      // pass C runs this many tiles behind pass A
+constexpr int kCbLag = 3;                      // pass C runs this many tiles behind pass A
 constexpr int kCbSlots = kCbLag + 1;           // slice-map, adjoint and TMEM slots
 constexpr int kCbScanners = 2;
 constexpr int kCbThreads = (kCbWarps + kCbScanners + 2) * 32;
