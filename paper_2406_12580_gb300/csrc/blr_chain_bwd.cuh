@@ -14,9 +14,10 @@
 //   producers (2 warps): one loads tile n's dh and rho into ring A; the other,
 //      a little before pass C needs it, tile n's x, rho and iota into ring C
 //      (rho is by then in L2), and once pass C has written the tile's outputs
-//      over them, sends those out by TMA store before refilling the stage. The first also writes each tile's decay
-//      constants and coordinates into a small ring of their own, so that the
-//      compute warps divide no tile index;
+//      over them, sends those out by TMA store before refilling the stage.
+//      The first also writes each tile's decay constants and coordinates into
+//      a small ring of their own, so that the compute warps divide no tile
+//      index;
 //   compute (kCbWarps warps, a slice of kCbSlice steps each, which starts at
 //      one of the forward's kept states): pass A of tile n evaluates the alphas
 //      of its slice and folds the reverse recurrence from a zero carry, last
@@ -52,9 +53,9 @@ constexpr int kCbThreads = (kCbWarps + kCbScanners + 2) * 32;
 constexpr uint32_t kCbTmemCols = 512;
 // Registers per thread, as kChainMaxRegs.
 constexpr int kCbMaxRegs = (16384 / (((kCbThreads / 32 + 3) / 4) * 32)) / 8 * 8;
-// Tiles' decay constants and coordinates, a ring indexed by tile: the ring-A producer writes
-// tile i's once pass A of tile i - kCbStagesA has freed its stage, and pass C
-// of tile i - kCbStagesA - kCbLag + 1 may still be to run.
+// Tiles' decay constants and coordinates, a ring indexed by tile: the ring-A
+// producer writes tile i's once pass A of tile i - kCbStagesA has freed its
+// stage, and pass C of tile i - kCbStagesA - kCbLag + 1 may still be to run.
 constexpr int kCbRates = 8;
 static_assert(kCbRates > kCbLag + kCbStagesA, "a tile's decay constants outlive its pass C");
 static_assert(kCbWarps * kCbSlice == kChainTile, "the backward tiles are the forward's");
@@ -88,8 +89,7 @@ struct ChainBwdSmem {
   static constexpr size_t poly = up(rates + (size_t)kCbRates * CHW * sizeof(float2));  // int [kCbRates]
   static constexpr size_t tmeta = up(poly + (size_t)kCbRates * sizeof(int));  // int4 [kCbRates]
   static constexpr size_t maps = up(tmeta + (size_t)kCbRates * sizeof(int4));  // float2 [MS][W][CHW]
-  static constexpr size_t meta = up(maps + (size_t)kCbSlots * kCbWarps * CHW * sizeof(float2));  // int4 [MS]
-  static constexpr size_t tmem = up(meta + (size_t)kCbSlots * sizeof(int4));
+  static constexpr size_t tmem = up(maps + (size_t)kCbSlots * kCbWarps * CHW * sizeof(float2));
   static constexpr size_t bars = up(tmem + sizeof(uint32_t));
   static constexpr size_t end =
       bars + (size_t)(2 * kCbStagesA + 2 * kCbStagesC + 2 * kCbSlots) * sizeof(uint64_t);
@@ -209,7 +209,6 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
   int* polys = reinterpret_cast<int*>(base + SM::poly);
   int4* tmeta = reinterpret_cast<int4*>(base + SM::tmeta);  // [kCbRates]: tile coordinates
   float2* maps = reinterpret_cast<float2*>(base + SM::maps);
-  int4* meta = reinterpret_cast<int4*>(base + SM::meta);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(base + SM::tmem);
   uint64_t* fullA = reinterpret_cast<uint64_t*>(base + SM::bars);
   uint64_t* emptyA = fullA + SA;
@@ -402,7 +401,6 @@ __global__ void __maxnreg__(kCbMaxRegs) chain_bwd_kernel(const __grid_constant__
           ws[v] = map_apply(mw.x, ws[v], mw.y);
         }
       }
-      if (lane == 0) meta[m] = c;
       mbar_arrive(&carry_ready[m]);
     }
   } else {

@@ -197,6 +197,40 @@ def test_empty_sequence_and_batch():
     blr_scan_fwd(Desc(0, 10, D), e, e, lam, None, e, None, None)  # B = 0: nothing to do
 
 
+def test_chained_optional_arguments():
+    """The chained kernels (one long bfloat16 row) with every optional pointer
+    NULL: no h0, h, h_last in the forward (carries only), no dh_last and dh0
+    in the backward; then the backward again on the same workspace, which
+    must give the same gradients (its records are emptied again each call)."""
+    from paper_2406_12580_gb300 import (FAMILY_SEGMENTED, Desc, blr_scan_bwd, blr_scan_family,
+                                        blr_scan_fwd)
+    from paper_2406_12580_gb300.device import ScanBuffers
+    cfg = I.ScanConfig("chained, optional arguments NULL", B=1, L=16500, D=72, io=I.BF16, seed=35)
+    desc = Desc(cfg.B, cfg.L, cfg.D, 1, cfg.c)
+    assert blr_scan_family(desc) == FAMILY_SEGMENTED
+    inp = I.make_scan_inputs(cfg)
+    assert inp.h0 is None and inp.dh_last is None
+    buf = ScanBuffers.from_inputs(inp)
+    buf.h.fill_(7.0)
+    blr_scan_fwd(buf.desc, buf.x, buf.gl, buf.lam, None, None, None, buf.ws)
+    blr_scan_bwd(buf.desc, buf.dh, None, buf.x, buf.gl, buf.lam, None, buf.dx, buf.dgl, buf.dlam,
+                 None, buf.ws)
+    torch.cuda.synchronize()
+    assert torch.all(buf.h == 7.0)  # h untouched
+    want = oracle_outputs(inp)
+    got = gpu_outputs(buf)
+    compare(inp, {k: got[k] for k in ("dx", "dgl", "dlam")},
+            {k: want[k] for k in ("dx", "dgl", "dlam")})
+    first = [buf.dx.clone(), buf.dgl.clone(), buf.dlam.clone()]
+    blr_scan_bwd(buf.desc, buf.dh, None, buf.x, buf.gl, buf.lam, None, buf.dx, buf.dgl, buf.dlam,
+                 None, buf.ws)
+    torch.cuda.synchronize()
+    # the look-back folds whichever predecessors have published, so a repeat may
+    # differ from the first call by one bfloat16 unit in the last place
+    for a, b in zip(first, [buf.dx, buf.dgl, buf.dlam]):
+        assert normwise(b.float().cpu().numpy(), a.float().cpu().numpy()) <= 2.0 ** -7
+
+
 def test_backward_without_forward_carries_is_reported():
     from paper_2406_12580_gb300 import (BLR_ERR_WORKSPACE, BLR_OK, Desc, blr_workspace_status)
     from paper_2406_12580_gb300.device import ScanBuffers
