@@ -2,8 +2,9 @@
 // (batch row, channel group) chains and long sequences, reading every input
 // once and writing every output once.
 //
-// A tile is kChainTile consecutive steps of one chain (a 128-byte row segment:
-// 32 float32 or 64 bfloat16 channels of one batch row). Tiles are numbered
+// The path is bfloat16 I/O. A tile is kChainTile consecutive steps of one
+// chain (64 bfloat16 channels of one batch row, a 128-byte row segment; a
+// lane owns 2 channels as one float pair). Tiles are numbered
 // time-major (tile = time block * chains + chain); block j of a cooperative
 // grid of G resident blocks (one per SM) takes tiles j, j + G, j + 2G, ..., so
 // a tile only ever waits on tiles of smaller number. The block's warps have
